@@ -63,6 +63,7 @@ def _bind(path: str):
     lib.or_dense.argtypes = [f64p, ctypes.c_long, f32p, f32p, ctypes.c_int, ctypes.c_int, f64p]
     lib.or_heads.argtypes = [f64p, ctypes.c_int, ctypes.c_double, f64p]
     lib.or_round_bf16.argtypes = [f32p, ctypes.POINTER(ctypes.c_uint16), ctypes.c_long]
+    lib.or_round_fp16.argtypes = [f32p, f32p, ctypes.c_long]
     lib.or_set_threads.argtypes = [ctypes.c_int]
     lib.or_max_threads.restype = ctypes.c_int
     return lib
@@ -106,10 +107,15 @@ def extract_patches(adc, nticks, hits, psize: int = PATCH, ds: int = DOWNSAMPLE,
 _WKEYS = ("conv_w", "conv_b", "fc1_w", "fc1_b", "fc2_w", "fc2_b", "cls_w", "cls_b", "mic_w", "mic_b")
 
 
-def forward(patches, weights: dict, dims: dict | None = None, emulate_bf16: bool = False,
+_EMULATE = {None: 0, "bf16": 1, "fp16": 2}
+
+
+def forward(patches, weights: dict, dims: dict | None = None, emulate: str | None = None,
             threads: int | None = None, lib=None):
     """Sec. 2.2 network on [n][P][P] float32 patches.  Returns (logits, scores),
-    each [n][NC+1] float64: softmax classes (track, em, none) then Michel."""
+    each [n][NC+1] float64: softmax classes (track, em, none) then Michel.
+    ``emulate`` = "bf16" or "fp16" rounds the operands of the conv and of
+    dense-1 to that format first (a diagnostic reference for 16-bit paths)."""
     lib = lib or load()
     d = dict(EMTK_DIMS if dims is None else dims)
     patches = _c(patches, np.float32).reshape(-1, d["P"], d["P"])
@@ -120,7 +126,7 @@ def forward(patches, weights: dict, dims: dict | None = None, emulate_bf16: bool
     if threads is not None:
         lib.or_set_threads(int(threads))
     rc = lib.or_forward(ctypes.byref(_Dims(**d)), _p(patches, ctypes.c_float), n,
-                        *[_p(w, ctypes.c_float) for w in ws], int(bool(emulate_bf16)),
+                        *[_p(w, ctypes.c_float) for w in ws], _EMULATE[emulate],
                         _p(logits, ctypes.c_double), _p(scores, ctypes.c_double))
     if rc != 0:
         raise ValueError(f"or_forward failed ({rc})")
@@ -171,6 +177,15 @@ def round_bf16(x, lib=None):
     x = _c(x, np.float32)
     out = np.zeros(x.shape, np.uint16)
     lib.or_round_bf16(_p(x, ctypes.c_float), _p(out, ctypes.c_uint16), x.size)
+    return out
+
+
+def round_fp16(x, lib=None):
+    """Round float32 values to IEEE binary16 (nearest, ties to even); returns float32."""
+    lib = lib or load()
+    x = _c(x, np.float32)
+    out = np.zeros(x.shape, np.float32)
+    lib.or_round_fp16(_p(x, ctypes.c_float), _p(out, ctypes.c_float), x.size)
     return out
 
 

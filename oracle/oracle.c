@@ -30,10 +30,11 @@
  *   - softmax outputs are ordered (track, em, none), then the Michel sigmoid.
  *
  * Precision: the patch cut is fp32 by definition (it must be reproduced bit
- * for bit); everything in the network is accumulated in double.  An optional
- * bf16-emulating mode rounds the operands (patch, conv weights, conv outputs
- * after ReLU, dense-1 weights) to bf16 before use; it is a diagnostic aid, not
- * the acceptance reference.
+ * for bit); everything in the network is accumulated in double.  Optional
+ * emulating modes round the operands of the two large contractions (patch,
+ * conv weights, conv outputs after ReLU, dense-1 weights) to bf16 or to fp16
+ * before use, the points where a 16-bit tensor-core path rounds; they are a
+ * diagnostic reference, not the definition.
  */
 #include <math.h>
 #include <stdint.h>
@@ -67,6 +68,37 @@ static float round_bf16_f(float x)
     u &= 0xFFFF0000u;
     memcpy(&x, &u, 4);
     return x;
+}
+
+/* Round a finite float to the nearest IEEE binary16 value (ties to even,
+ * gradual underflow, overflow to infinity); returned as a float. */
+static float round_fp16_f(float x)
+{
+    if (x == 0.0f || !isfinite(x))
+        return x;
+    const float a = fabsf(x);
+    int e;
+    frexpf(a, &e);              /* a in [2^(e-1), 2^e) */
+    int qexp = e - 11;          /* 11 significant bits */
+    if (qexp < -24)
+        qexp = -24;             /* subnormal spacing 2^-24 */
+    const float q = ldexpf(1.0f, qexp);
+    float r = rintf(a / q) * q; /* a / q is exact: q is a power of two */
+    if (r >= 65520.0f)
+        r = INFINITY;
+    return copysignf(r, x);
+}
+
+void or_round_fp16(const float *in, float *out, long n)
+{
+    for (long i = 0; i < n; ++i)
+        out[i] = round_fp16_f(in[i]);
+}
+
+/* emulation modes: 0 none, 1 bf16, 2 fp16 */
+static float round_mode(float x, int mode)
+{
+    return mode == 1 ? round_bf16_f(x) : mode == 2 ? round_fp16_f(x) : x;
 }
 
 void or_round_bf16(const float *in, uint16_t *out, long n)
@@ -214,20 +246,21 @@ void or_heads(const double *logits, int NC, double logit_m, double *scores)
 /* Full network on n patches [n][P][P] (fp32).  Weights in the layouts of the
  * header comment, fp32.  Outputs (each [n][NC+1], double): the logits (NC
  * class logits then the Michel logit) and the scores (softmax then sigmoid).
- * emulate_bf16 != 0 rounds patch, conv weights, post-ReLU conv outputs and
- * dense-1 weights to bf16 before use. */
+ * emulate = 1 (bf16) or 2 (fp16) rounds patch, conv weights, post-ReLU conv
+ * outputs and dense-1 weights to that format before use; 0 rounds nothing. */
 int or_forward(const or_dims *d, const float *patches, long n,
                const float *conv_w, const float *conv_b,
                const float *fc1_w, const float *fc1_b,
                const float *fc2_w, const float *fc2_b,
                const float *cls_w, const float *cls_b,
                const float *mic_w, const float *mic_b,
-               int emulate_bf16, double *logits, double *scores)
+               int emulate, double *logits, double *scores)
 {
     if (!d || n < 0)
         return OR_ERR_ARG;
     const int P = d->P, R = d->R, F = d->F, N1 = d->N1, N2 = d->N2, NC = d->NC;
-    if (P <= 0 || R <= 0 || R > P || F <= 0 || N1 <= 0 || N2 <= 0 || NC <= 0)
+    if (P <= 0 || R <= 0 || R > P || F <= 0 || N1 <= 0 || N2 <= 0 || NC <= 0 ||
+        emulate < 0 || emulate > 2)
         return OR_ERR_ARG;
     if (n == 0)
         return OR_OK;
@@ -244,11 +277,11 @@ int or_forward(const or_dims *d, const float *patches, long n,
         return OR_ERR_OOM;
     }
     for (int i = 0; i < R * R * F; ++i)
-        cw[i] = emulate_bf16 ? (double)round_bf16_f(conv_w[i]) : (double)conv_w[i];
+        cw[i] = (double)round_mode(conv_w[i], emulate);
     for (int f = 0; f < F; ++f)
         cb[f] = conv_b[f];
     const float *W1 = fc1_w;
-    if (emulate_bf16) {
+    if (emulate) {
         w1 = (float *)malloc(sizeof(float) * K1 * N1);
         if (!w1) {
             free(cw);
@@ -256,7 +289,7 @@ int or_forward(const or_dims *d, const float *patches, long n,
             return OR_ERR_OOM;
         }
         for (long i = 0; i < K1 * N1; ++i)
-            w1[i] = round_bf16_f(fc1_w[i]);
+            w1[i] = round_mode(fc1_w[i], emulate);
         W1 = w1;
     }
 
@@ -276,11 +309,11 @@ int or_forward(const or_dims *d, const float *patches, long n,
             for (long h = 0; h < n; ++h) {
                 const float *p = patches + h * (long)P * P;
                 for (int i = 0; i < P * P; ++i)
-                    img[i] = emulate_bf16 ? (double)round_bf16_f(p[i]) : (double)p[i];
+                    img[i] = (double)round_mode(p[i], emulate);
                 or_conv_relu(img, P, cw, cb, R, F, act);
-                if (emulate_bf16)
+                if (emulate)
                     for (long k = 0; k < K1; ++k)
-                        act[k] = (double)round_bf16_f((float)act[k]);
+                        act[k] = (double)round_mode((float)act[k], emulate);
                 or_dense(act, K1, W1, fc1_b, N1, 1, h1);
                 or_dense(h1, N1, fc2_w, fc2_b, N2, 1, h2);
                 or_dense(h2, N2, cls_w, cls_b, NC, 0, z);

@@ -271,6 +271,18 @@ def pin_bf16_rounding(lib):
     assert np.array_equal(got, want)
 
 
+def pin_fp16_rounding(lib):
+    rng = np.random.default_rng(13)
+    x = np.concatenate([(rng.standard_normal(4000) * 100).astype(np.float32),
+                        (rng.standard_normal(1000) * 1e-5).astype(np.float32),
+                        np.array([1.0 + 2.0 ** -11, 1.0 + 3 * 2.0 ** -11, 65504.0, 65519.0, 65520.0,
+                                  -70000.0, 2.0 ** -25, 3 * 2.0 ** -26, 1e-30, 0.0], np.float32)])
+    got = oracle.round_fp16(x, lib=lib)
+    with np.errstate(over="ignore"):
+        want = x.astype(np.float16).astype(np.float32)
+    assert np.array_equal(got.view(np.uint32), want.view(np.uint32))
+
+
 def pin_transmit_volume(lib):
     bits = FACTS["patches_per_event"] * FACTS["patch_side"] ** 2 * FACTS["bits_per_pixel"]
     assert abs(bits / 1e9 - FACTS["transmit_gbit_per_event"]) < 0.06
@@ -279,7 +291,7 @@ def pin_transmit_volume(lib):
 PINS = [pin_parameter_count, pin_conv_shape, pin_constant_plane, pin_ramps, pin_impulse,
         pin_outside_and_partial, pin_negative_ticks, pin_patches_brute_force, pin_conv_library,
         pin_dense_library, pin_heads, pin_forward_library, pin_forward_full_size, pin_zero_weights,
-        pin_flatten_order, pin_bf16_rounding, pin_transmit_volume]
+        pin_flatten_order, pin_bf16_rounding, pin_fp16_rounding, pin_transmit_volume]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=[p.__name__ for p in PINS])
@@ -287,20 +299,25 @@ def test_pin(pin, oracle_lib):
     pin(oracle_lib)
 
 
-def test_emulated_bf16_is_rounding_only(oracle_lib):
-    """The bf16-emulating mode equals the plain mode on inputs that are already
-    bf16 values with activations that need no rounding (one-filter identity
-    conv on bf16 patches, bf16 weights)."""
+@pytest.mark.parametrize("mode", ["bf16", "fp16"])
+def test_emulated_mode_is_rounding_only(mode, oracle_lib):
+    """An emulating mode equals the plain mode on inputs that are already
+    values of that format with activations that need no rounding (one-filter
+    identity conv on rounded patches, rounded weights)."""
+    rnd = (lambda a: (oracle.round_bf16(a).astype(np.uint32) << 16).view(np.float32).reshape(a.shape)) \
+        if mode == "bf16" else (lambda a: oracle.round_fp16(a))
     rng = np.random.default_rng(12)
     d = dict(P=6, R=1, F=1, N1=4, N2=3, NC=3)
     wt = synth.he_normal_weights(5, bias_std=0.1, dims=d)
     wt["conv_w"][:] = 1.0
     wt["conv_b"][:] = 0.0
-    wt["fc1_w"] = (oracle.round_bf16(wt["fc1_w"]).astype(np.uint32) << 16).view(np.float32).reshape(wt["fc1_w"].shape)
-    x = (oracle.round_bf16((rng.standard_normal((4, 6, 6)) * 5).astype(np.float32)).astype(np.uint32) << 16).view(np.float32)
+    wt["fc1_w"] = rnd(wt["fc1_w"])
+    x = rnd((rng.standard_normal((4, 6, 6)) * 5).astype(np.float32))
     a = oracle.forward(x, wt, dims=d)
-    b = oracle.forward(x, wt, dims=d, emulate_bf16=True)
+    b = oracle.forward(x, wt, dims=d, emulate=mode)
     assert np.array_equal(a[0], b[0])
+    c = oracle.forward((rng.standard_normal((4, 6, 6)) * 5).astype(np.float32), wt, dims=d, emulate=mode)
+    assert np.all(np.isfinite(c[1]))
 
 
 # ---------------------------------------------------------- planted mistakes
