@@ -1,0 +1,366 @@
+"""Benchmark: EmTrackMichelId hit identification on GB300.
+
+One step = one pass of the whole hot path over one synthetic event: the
+patch cut (time-interval image + gather), the fused conv + dense-1 tensor-core
+kernel and the dense-2/heads kernel, for all 18 planes of a full 6-APA event
+(15,360 wires x 6000 ticks, 60,000 hits) in one batched call
+(emtk_infer_batch), bf16.  Inputs are device-resident when a timed step
+starts; L2 is flushed (256 MiB write) between timed steps.
+
+Prints one JSON line (rank 0).  `--impl reference` times the CPU oracle on
+the host cores instead, on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2009_04509_gb300 import synth  # noqa: E402
+
+FLOP_CONV = 2 * 44 * 44 * 48 * 25          # 4,646,400 per hit (25 taps)
+FLOP_FC1 = 2 * 92928 * 128                  # 23,789,568
+FLOP_TAIL = 2 * (128 * 32 + 32 * 4)         # 8,448
+FLOP_PER_HIT = FLOP_CONV + FLOP_FC1 + FLOP_TAIL  # 28,444,416
+METRIC = "hit patches/sec on 1 GB300 (extract+CNN); % bf16 tensor peak; gather HBM GB/s"
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return dict(hbm=d["hbm_gbs"], bf16=d["bf16_tflops"], bf16_sus=d.get("bf16_tflops_sustained", d["bf16_tflops"]),
+                    source="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, source="fallback")
+
+
+def window_union_bytes(planes, patch=48, ds=6):
+    """Bytes of ADC inside the union of all hits' patch windows (48 wires x
+    48 intervals of 6 ticks), clipped to the plane, each sample counted once:
+    the least the patch cut has to read."""
+    total = 0
+    half = patch // 2
+    for p in planes:
+        nint = p.nticks // ds
+        cover = np.zeros((p.nwires + 1, nint + 1), np.int32)
+        if p.nhits:
+            w0 = np.clip(p.hits[:, 0].astype(np.int64) - half, 0, p.nwires)
+            w1 = np.clip(p.hits[:, 0].astype(np.int64) + half, 0, p.nwires)
+            b = np.floor_divide(p.hits[:, 1].astype(np.int64), ds)
+            b0 = np.clip(b - half, 0, nint)
+            b1 = np.clip(b + half, 0, nint)
+            np.add.at(cover, (w0, b0), 1)
+            np.add.at(cover, (w1, b0), -1)
+            np.add.at(cover, (w0, b1), -1)
+            np.add.at(cover, (w1, b1), 1)
+        cov = np.cumsum(np.cumsum(cover, 0), 1)[: p.nwires, :nint] > 0
+        total += int(cov.sum()) * ds * 4
+    return total
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms."""
+    Q = ("index,uuid,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid: str | None):
+        self.uuid = uuid
+        self.proc = None
+        self.path = os.path.join("/tmp", f"emtk_clocks_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                                          "-lms", "200"], stdout=self.f, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.f.close()
+        rows = []
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 10:
+                continue
+            if self.uuid and self.uuid not in parts[1]:
+                continue
+            rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        mx = [float(r[3]) for r in rows if r[3].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[6 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+def gpu_uuid():
+    import torch
+    try:
+        u = str(torch.cuda.get_device_properties(torch.cuda.current_device()).uuid)
+        return u if u.startswith("GPU-") else "GPU-" + u
+    except Exception:
+        return None
+
+
+# ------------------------------------------------------------- CPU oracle
+def cpu_oracle_rate(planes, weights, budget_s: float = 15.0):
+    """Oracle hits/s on the host cores: the patch cut of every hit of the
+    event, then the network on as many hits as fit the time budget."""
+    import oracle
+    oracle.build()
+    lib = oracle.load()
+    threads = oracle.max_threads(lib)
+    t0 = time.perf_counter()
+    nh = 0
+    patches = []
+    for p in planes:
+        patches.append(oracle.extract_patches(p.adc, p.nticks, p.hits, lib=lib))
+        nh += p.nhits
+    t_cut = time.perf_counter() - t0
+    allp = np.concatenate(patches)
+    rng = np.random.default_rng(0)
+    idx = rng.permutation(allp.shape[0])
+    done, t_net, chunk = 0, 0.0, 4 * threads
+    while t_net < budget_s and done < allp.shape[0]:
+        sel = idx[done: done + chunk]
+        t1 = time.perf_counter()
+        oracle.forward(allp[sel], weights, lib=lib)
+        t_net += time.perf_counter() - t1
+        done += sel.size
+    per_hit = t_cut / nh + t_net / done
+    return 1.0 / per_hit, threads, (f"patch cut of all {nh} hits ({t_cut:.2f} s) + network (fp64) on "
+                                    f"{done} random hits ({t_net:.2f} s), {threads} OpenMP threads")
+
+
+# -------------------------------------------------------------------- main
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="emtk", choices=["emtk", "reference"])
+    ap.add_argument("--workload", default="full_event", choices=["full_event", "apa"])
+    ap.add_argument("--precision", default="bf16", choices=["bf16", "fp16", "fp32"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-budget", type=float, default=15.0)
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        return run_reference(args, rank, world)
+
+    import torch
+    torch.cuda.set_device(local_rank)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+
+    from paper_2009_04509_gb300 import emtk
+    planes = synth.full_event(seed=rank) if args.workload == "full_event" else synth.apa(seed=rank)
+    weights = synth.he_normal_weights(0)
+    nhits = sum(p.nhits for p in planes)
+    dev = torch.device("cuda", local_rank)
+    adc = [torch.from_numpy(p.adc).to(dev) for p in planes]
+    hits = [torch.from_numpy(p.hits).to(dev) for p in planes]
+    scores = [torch.empty((p.nhits, 4), dtype=torch.float32, device=dev) for p in planes]
+    items = [(a, p.nticks, h, s) for a, p, h, s in zip(adc, planes, hits, scores)]
+    ctx = emtk.emtk_create(weights, precision=args.precision, device=local_rank, profile=True)
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        if args.workload == "full_event":
+            emtk.emtk_infer_batch(ctx, items, stream)
+        else:
+            for it in items:
+                emtk.emtk_infer(ctx, it[0], it[1], it[2], it[3], stream)
+
+    for _ in range(args.warmup):
+        step()
+    assert emtk.emtk_check(ctx, stream) == emtk.EMTK_OK
+    base = emtk.emtk_get_stats(ctx)
+
+    clocks = ClockSampler(gpu_uuid())
+    clocks.start()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    for i in range(args.steps):
+        flush.zero_()
+        ev[i][0].record(stream)
+        step()
+        ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    clk = clocks.stop()
+    rc = emtk.emtk_check(ctx, stream)
+    assert rc == emtk.EMTK_OK, emtk.status_string(rc)
+    st = emtk.emtk_get_stats(ctx)
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    total_ms = float(sum(step_ms))
+    if dist:
+        t = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    ms_per_step = total_ms / args.steps
+    value = world * nhits * args.steps / (total_ms / 1e3)
+
+    kms = {k: st["kernel_ms"][k] - base["kernel_ms"][k] for k in emtk.KERNELS}
+    kn = {k: st["kernel_launches"][k] - base["kernel_launches"][k] for k in emtk.KERNELS}
+    launches = st["launches"] - base["launches"]
+    peaks = load_peaks()
+    net_ms = kms["network"] / max(1, kn["network"])
+    hits_per_launch = nhits * args.steps / max(1, kn["network"])
+    flop_net = (FLOP_CONV + FLOP_FC1) * hits_per_launch
+    achieved = flop_net / (net_ms / 1e3) / 1e12
+    union = window_union_bytes(planes)
+    patch_bytes = nhits * 48 * 48 * (4 if args.precision == "fp32" else 2)
+    cut_ms = (kms["intervals"] + kms["gather"]) / args.steps
+    cut_gbs = (union + patch_bytes) / (cut_ms / 1e3) / 1e9
+
+    # end to end through the public call: host planes and hits in, scores out
+    e2e = None
+    if rank == 0 or world > 1:
+        e2e = measure_e2e(emtk, ctx, planes, dev, stream, args, torch)
+
+    out = {
+        "metric": METRIC,
+        "value": value,
+        "unit": "hits/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": ms_per_step,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": args.precision,
+        "data": "synthetic (seeded ProtoDUNE-SP-shaped planes and hits; He-normal seed-0 weights)",
+        "config": {"workload": ("full 6-APA event: 18 planes (800/800/960 wires) x 6000 ticks, 60,000 hits, "
+                                "one emtk_infer_batch") if args.workload == "full_event" else
+                   "one APA: planes 800/800/480 x 6000 ticks, 20,000 hits, one emtk_infer per plane",
+                   "hits_per_step": nhits, "planes": len(planes), "precision": args.precision,
+                   "l2": "flushed between steps (256 MiB write); planes (368.6 MB) exceed L2",
+                   "parallelism": f"replicas x{world} (independent events, no collective)"},
+        "gpu_launches": launches,
+        "roofline": {"bound": "tensor", "kernel": "cnn_tc_kernel (conv 5x5x48 + dense-1, tcgen05)"
+                     if args.precision != "fp32" else "cnn_fp32_kernel",
+                     "achieved": achieved, "peak": peaks["bf16_sus"], "unit": "TFLOP/s",
+                     "frac": achieved / peaks["bf16_sus"],
+                     "peak_source": f"{peaks['source']} bf16 sustained", "frac_of_burst": achieved / peaks["bf16"],
+                     "flop_per_hit": FLOP_CONV + FLOP_FC1, "hits_per_launch": hits_per_launch,
+                     "launch_ms": net_ms, "traffic": None},
+        "extraction": {"bound": "hbm", "achieved": cut_gbs, "peak": peaks["hbm"], "unit": "GB/s",
+                       "frac": cut_gbs / peaks["hbm"], "algorithmic_bytes": union + patch_bytes,
+                       "ms_per_step": cut_ms},
+        "kernel_ms_per_step": {k: v / args.steps for k, v in kms.items()},
+        "whole_step_frac_of_bf16_peak": value * FLOP_PER_HIT / 1e12 / peaks["bf16"] / world,
+        "clocks": clk,
+    }
+    if e2e:
+        out["e2e"] = e2e
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        rate, cores, sample = cpu_oracle_rate(planes, weights, args.cpu_budget)
+        out["cpu_baseline"] = {"value": rate, "unit": "hits/s", "cores": cores, "kind": "oracle", "sample": sample}
+    emtk.emtk_destroy(ctx)
+    if rank == 0:
+        print(json.dumps(out))
+    if dist:
+        dist.destroy_process_group()
+
+
+def measure_e2e(emtk, ctx, planes, dev, stream, args, torch):
+    """Same metric through the public call with host buffers: every step
+    copies the planes and hits from pinned host memory, runs the batch and
+    reads the scores back."""
+    h_adc = [torch.from_numpy(p.adc).pin_memory() for p in planes]
+    h_hits = [torch.from_numpy(p.hits).pin_memory() for p in planes]
+    h_sc = [torch.empty((p.nhits, 4), dtype=torch.float32).pin_memory() for p in planes]
+    d_adc = [torch.empty_like(a, device=dev) for a in h_adc]
+    d_hits = [torch.empty_like(h, device=dev) for h in h_hits]
+    d_sc = [torch.empty_like(s, device=dev) for s in h_sc]
+    items = [(a, p.nticks, h, s) for a, p, h, s in zip(d_adc, planes, d_hits, d_sc)]
+    nhits = sum(p.nhits for p in planes)
+    steps = max(3, min(args.steps, 20))
+
+    def one():
+        for d, h in zip(d_adc, h_adc):
+            d.copy_(h, non_blocking=True)
+        for d, h in zip(d_hits, h_hits):
+            d.copy_(h, non_blocking=True)
+        emtk.emtk_infer_batch(ctx, items, stream)
+        for h, d in zip(h_sc, d_sc):
+            h.copy_(d, non_blocking=True)
+
+    for _ in range(3):
+        one()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(steps):
+        one()
+    b.record(stream)
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / steps
+    h2d = sum(x.numel() * x.element_size() for x in h_adc + h_hits)
+    d2h = sum(x.numel() * x.element_size() for x in h_sc)
+    return {"value": nhits / (ms / 1e3), "unit": "hits/s", "ms_per_step": ms, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "steps": steps}
+
+
+def run_reference(args, rank, world):
+    """The oracle on the host cores, on the same workload, each step a
+    bounded sample of it."""
+    if rank != 0:
+        return
+    planes = synth.full_event(seed=0) if args.workload == "full_event" else synth.apa(seed=0)
+    weights = synth.he_normal_weights(0)
+    budget = max(1.0, min(args.cpu_budget, 120.0 / max(1, args.steps + args.warmup)))
+    rates = []
+    sample = ""
+    cores = 0
+    for i in range(args.warmup + args.steps):
+        rate, cores, sample = cpu_oracle_rate(planes, weights, budget)
+        if i >= args.warmup:
+            rates.append(rate)
+    value = float(statistics.median(rates))
+    nh = sum(p.nhits for p in planes)
+    out = {"impl": "reference", "metric": METRIC, "value": value, "unit": "hits/s", "n_gpus": world,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": nh / value * 1e3, "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "config": {"workload": "full 6-APA event: 18 planes x 6000 ticks, 60,000 hits (CPU oracle, sampled)"},
+           "cpu_baseline": {"value": value, "unit": "hits/s", "cores": cores, "kind": "oracle", "sample": sample},
+           "e2e": {"value": value, "unit": "hits/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out))
+
+
+if __name__ == "__main__":
+    main()

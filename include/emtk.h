@@ -1,0 +1,192 @@
+/*
+ * emtk.h -- C ABI of the GB300 EmTrackMichelId hit-identification library.
+ *
+ * The library computes, on one GPU, what arXiv:2009.04509 offloads to its
+ * inference servers: for every reconstructed wire hit, a 48x48 patch of
+ * deconvolved charge (rows = wires, columns = time intervals of 6 ticks) is
+ * cut around the hit (Sec. 2.1), and the EmTrackMichelId network scores it
+ * (Sec. 2.2): conv 5x5 with 48 filters + ReLU, dense 128 + ReLU, dense 32 +
+ * ReLU, a 3-way softmax (track, em, none) and a 1-way sigmoid (Michel).
+ *
+ * Conventions for every entry point below:
+ *   - Pointers named d_* are device memory owned by the caller.  They must
+ *     stay valid until the work enqueued on the caller's stream completes.
+ *   - All work is enqueued on the caller's stream; nothing synchronises
+ *     unless stated.  A context may be used from one stream at a time.
+ *   - Argument errors are reported synchronously and enqueue nothing.
+ *     Launch failures return EMTK_ERR_CUDA.  A device-side wait that gave up
+ *     (EMTK_ERR_TIMEOUT) is reported by emtk_check().
+ *   - For a fixed precision and fixed sizes, results are bit-identical from
+ *     run to run.
+ *   - Every hit coordinate is valid: pixels that fall outside the plane are
+ *     zero, so a hit far outside the plane gets an all-zero patch.
+ */
+#ifndef EMTK_H
+#define EMTK_H
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define EMTK_API __attribute__((visibility("default")))
+#else
+#define EMTK_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as the CUDA runtime's cudaStream_t; NULL is the legacy default
+ * stream. */
+typedef struct CUstream_st *emtk_stream;
+
+typedef struct emtk_ctx emtk_ctx;
+
+typedef enum {
+    EMTK_OK = 0,
+    EMTK_ERR_ARG = 1,         /* null pointer, negative size, bad enum, ... */
+    EMTK_ERR_ALIGN = 2,       /* d_adc not 16-byte aligned or ld % 4 != 0 */
+    EMTK_ERR_OOM = 3,         /* device allocation failed */
+    EMTK_ERR_CUDA = 4,        /* a CUDA call or launch failed */
+    EMTK_ERR_TIMEOUT = 5,     /* a bounded device-side wait gave up */
+    EMTK_ERR_UNSUPPORTED = 6  /* precision or device not supported */
+} emtk_status;
+
+/* Arithmetic of the network.
+ *   EMTK_FP32: fp32 operands, fp32 accumulation (CUDA cores).
+ *   EMTK_BF16: bf16 patch, conv weights, conv activations and dense-1
+ *              weights; fp32 accumulation on the tcgen05 tensor cores;
+ *              dense-2 and heads in fp32.
+ *   EMTK_FP16: as EMTK_BF16 with IEEE fp16 operands (same tensor rate,
+ *              8x finer rounding; activations above 65504 saturate).
+ *   EMTK_TF32: reserved; emtk_create returns EMTK_ERR_UNSUPPORTED. */
+typedef enum { EMTK_FP32 = 0, EMTK_TF32 = 1, EMTK_BF16 = 2, EMTK_FP16 = 3 } emtk_precision;
+
+/* Element type of a patch buffer. */
+typedef enum { EMTK_PATCH_F32 = 0, EMTK_PATCH_BF16 = 1, EMTK_PATCH_F16 = 2 } emtk_patch_format;
+
+/* A reconstructed hit: wire index in the plane and raw tick index of its
+ * peak time (Sec. 2.1).  The hit's time interval is floor(tick / 6). */
+typedef struct {
+    int32_t wire;
+    int32_t tick;
+} emtk_hit;
+
+/* Network weights, host fp32, copied and converted by emtk_create (Sec. 2.2;
+ * 11,900,420 values in total):
+ *   conv_w [5][5][1][48]  tap row i, tap column j, input channel, filter
+ *   conv_b [48]
+ *   fc1_w  [92928][128]   row index (y*44 + x)*48 + c: conv map c at (y, x)
+ *   fc1_b  [128]
+ *   fc2_w  [128][32]   fc2_b [32]
+ *   cls_w  [32][3]     cls_b [3]    softmax logits (track, em, none)
+ *   mic_w  [32][1]     mic_b [1]    Michel logit */
+typedef struct {
+    const float *conv_w, *conv_b, *fc1_w, *fc1_b, *fc2_w, *fc2_b, *cls_w, *cls_b, *mic_w, *mic_b;
+} emtk_weights;
+
+/* Creation options; emtk_create(w, NULL, ...) uses the defaults in brackets.
+ *   precision       [EMTK_BF16]
+ *   max_hits        hits processed per internal chunk; sizes the workspace
+ *                   [65536]; larger calls are processed in chunks
+ *   debug_logits    0: d_scores is [n][4]; 1: d_scores is [n][8], the 4
+ *                   scores followed by the 4 logits [0]
+ *   wait_timeout_ns limit of every device-side wait in the tensor-core
+ *                   kernel, in nanoseconds [2e9]
+ *   debug_stall     test knob: 1 makes the tensor-core kernel wait once on
+ *                   a barrier nothing arrives at, so the wait runs out and
+ *                   the call's emtk_check reports EMTK_ERR_TIMEOUT [0]
+ *   profile         1: bracket every kernel launch with CUDA events on the
+ *                   caller's stream; emtk_get_stats then reports device time
+ *                   per kernel [0] */
+typedef struct {
+    emtk_precision precision;
+    int32_t max_hits;
+    int32_t debug_logits;
+    int64_t wait_timeout_ns;
+    int32_t debug_stall;
+    int32_t profile;
+} emtk_options;
+
+/* One client request for emtk_infer_batch: a plane and its hits. */
+typedef struct {
+    const float *d_adc;       /* [nwires][ld] fp32, 16-byte aligned, ld % 4 == 0 */
+    int32_t nwires, nticks;
+    int64_t ld;
+    const emtk_hit *d_hits;   /* [nhits] */
+    int32_t nhits;
+    float *d_scores;          /* [nhits][4] (or [nhits][8] with debug_logits) */
+} emtk_request;
+
+/* Kernel classes of the hot path, for per-kernel timing. */
+typedef enum {
+    EMTK_KERNEL_INTERVALS = 0, /* plane -> time-interval image */
+    EMTK_KERNEL_GATHER = 1,    /* interval image -> 48x48 patches */
+    EMTK_KERNEL_NETWORK = 2,   /* conv + dense-1 (tensor cores or fp32) */
+    EMTK_KERNEL_HEAD = 3,      /* dense-1 sum + dense-2 + heads */
+    EMTK_KERNEL_CONVERT = 4,   /* fp32 patches -> 16 bit (emtk_infer_patches) */
+    EMTK_NUM_KERNELS = 5
+} emtk_kernel;
+
+typedef struct {
+    uint64_t calls, hits, launches, chunks;
+    uint64_t batch_hist[8];   /* hits per launch: <256, <1k, <2k, <4k, <8k, <16k, <64k, >=64k */
+    /* with options.profile: launches and summed device milliseconds per
+     * kernel class (emtk_get_stats waits for the recorded events) */
+    uint64_t kernel_launches[EMTK_NUM_KERNELS];
+    double kernel_ms[EMTK_NUM_KERNELS];
+} emtk_stats;
+
+/* Fills *out with the defaults listed above. */
+EMTK_API void emtk_default_options(emtk_options *out);
+
+/* Creates a context on CUDA device `device`: uploads and converts the
+ * weights and allocates the workspace.  Returns EMTK_ERR_UNSUPPORTED for
+ * EMTK_TF32 or a device older than compute capability 10.3 when a
+ * tensor-core precision is asked for.  *out is NULL on failure. */
+EMTK_API emtk_status emtk_create(const emtk_weights *w, const emtk_options *opt, int device, emtk_ctx **out);
+
+/* Frees the context (synchronises its device first).  NULL is accepted. */
+EMTK_API emtk_status emtk_destroy(emtk_ctx *ctx);
+
+/* Scores every hit of one plane (Sec. 2.1 + 2.2).
+ *   d_adc    [nwires][ld] fp32 deconvolved charge, nticks valid ticks per
+ *            row; 16-byte aligned, ld % 4 == 0 and ld >= nticks
+ *   d_hits   [nhits]
+ *   d_scores [nhits][4] = {p_track, p_em, p_none, p_michel} (fp32)
+ * nhits == 0 returns EMTK_OK and enqueues nothing. */
+EMTK_API emtk_status emtk_infer(emtk_ctx *ctx, const float *d_adc, int32_t nwires, int32_t nticks, int64_t ld,
+                       const emtk_hit *d_hits, int32_t nhits, float *d_scores, emtk_stream stream);
+
+/* Request batching: concatenates the hit lists of `nreq` requests (a host
+ * array; each request has its own plane and output) and scores them in one
+ * pass of the hot path.  This stands in for the inference server's dynamic
+ * batching (Sec. 3.2).  Requests with nhits == 0 are allowed. */
+EMTK_API emtk_status emtk_infer_batch(emtk_ctx *ctx, const emtk_request *reqs, int32_t nreq, emtk_stream stream);
+
+/* Patch cut only (Sec. 2.1): d_patches [nhits][48][48] of `fmt`.  F32 is the
+ * exact fp32 value; BF16 / F16 are that value rounded to nearest-even. */
+EMTK_API emtk_status emtk_extract_patches(emtk_ctx *ctx, const float *d_adc, int32_t nwires, int32_t nticks,
+                                 int64_t ld, const emtk_hit *d_hits, int32_t nhits, void *d_patches,
+                                 emtk_patch_format fmt, emtk_stream stream);
+
+/* Network only (Sec. 2.2) on pre-cut fp32 patches [n][48][48] -> d_scores. */
+EMTK_API emtk_status emtk_infer_patches(emtk_ctx *ctx, const float *d_patches, int32_t n, float *d_scores,
+                               emtk_stream stream);
+
+/* Synchronises `stream`, then reports (and clears) the context's device
+ * status: EMTK_ERR_TIMEOUT if a device-side wait gave up since the last
+ * check, EMTK_ERR_CUDA on a sticky CUDA error, else EMTK_OK. */
+EMTK_API emtk_status emtk_check(emtk_ctx *ctx, emtk_stream stream);
+
+/* Counters since creation.  In profile mode this first waits for the events
+ * of every launch not yet read back. */
+EMTK_API emtk_status emtk_get_stats(emtk_ctx *ctx, emtk_stats *out);
+
+/* Static English text for a status code. */
+EMTK_API const char *emtk_status_string(emtk_status s);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* EMTK_H */

@@ -1,0 +1,463 @@
+// C ABI of the library (include/emtk.h): argument checks, workspace, the
+// hot-path sequence and counters.  Every launch goes to the caller's stream.
+#include <cuda.h>
+
+#include <algorithm>
+#include <cstdlib>
+#include <cstring>
+#include <new>
+
+#include "emtk_internal.h"
+
+using namespace emtk;
+
+namespace {
+
+struct DeviceGuard {  // restores the caller's current device
+    int prev = -1;
+    bool ok = false;
+    explicit DeviceGuard(int dev) {
+        if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+        ok = cudaSetDevice(dev) == cudaSuccess;
+    }
+    ~DeviceGuard() {
+        if (prev >= 0) cudaSetDevice(prev);
+    }
+};
+
+bool tensor_precision(emtk_precision p) { return p == EMTK_BF16 || p == EMTK_FP16; }
+
+emtk_patch_format patch_format(emtk_precision p) {
+    return p == EMTK_BF16 ? EMTK_PATCH_BF16 : p == EMTK_FP16 ? EMTK_PATCH_F16 : EMTK_PATCH_F32;
+}
+
+size_t patch_elem_bytes(emtk_patch_format f) { return f == EMTK_PATCH_F32 ? 4 : 2; }
+
+int out_stride(const emtk_ctx *c) { return c->opt.debug_logits ? 8 : 4; }
+
+int n_pad_of(int n) { return (n + 127) / 128 * 128; }
+
+constexpr int64_t kPartialCap = 64ll * 1024 * 1024;  // floats of the partial-sum workspace
+
+template <typename T>
+cudaError_t dmalloc(T **p, size_t bytes) {
+    void *v = nullptr;
+    cudaError_t e = cudaMalloc(&v, bytes);
+    *p = static_cast<T *>(v);
+    return e;
+}
+
+template <typename T>
+cudaError_t upload(T **p, const float *src, size_t n) {
+    cudaError_t e = dmalloc(p, n * sizeof(float));
+    if (e != cudaSuccess) return e;
+    return cudaMemcpy(*p, src, n * sizeof(float), cudaMemcpyHostToDevice);
+}
+
+void drain_events(emtk_ctx *c);
+
+void free_ctx(emtk_ctx *c) {
+    if (!c) return;
+    drain_events(c);
+    DeviceWeights &w = c->w;
+    for (void *p : {(void *)w.conv_w, (void *)w.conv_b, (void *)w.fc1_w, (void *)w.fc1_b, (void *)w.fc2_w,
+                    (void *)w.fc2_b, (void *)w.cls_w, (void *)w.cls_b, (void *)w.mic_w, (void *)w.mic_b,
+                    (void *)w.w1_tiles, (void *)w.convB, c->ws.dimg, c->ws.patches, (void *)c->ws.dest,
+                    (void *)c->ws.partials, (void *)c->ws.status})
+        if (p) cudaFree(p);
+    delete static_cast<CUtensorMap *>(w.w1_tmap);
+    delete c;
+}
+
+emtk_status cuda_status(cudaError_t e) {
+    if (e == cudaSuccess) return EMTK_OK;
+    if (e == cudaErrorMemoryAllocation) return EMTK_ERR_OOM;
+    return EMTK_ERR_CUDA;
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+emtk_status check_plane(const float *d_adc, int32_t nwires, int32_t nticks, int64_t ld, const emtk_hit *d_hits,
+                        int32_t nhits) {
+    if (nwires < 0 || nticks < 0 || nhits < 0 || ld < nticks) return EMTK_ERR_ARG;
+    if (nhits > 0 && (d_hits == nullptr || d_adc == nullptr)) return EMTK_ERR_ARG;
+    if (d_adc != nullptr && (!aligned16(d_adc) || (ld % 4) != 0)) return EMTK_ERR_ALIGN;
+    if ((reinterpret_cast<uintptr_t>(d_hits) & 7u) != 0) return EMTK_ERR_ALIGN;
+    return EMTK_OK;
+}
+
+// Profile mode: events around one launch on the caller's stream.
+struct Prof {
+    emtk_ctx *c;
+    int kind;
+    cudaStream_t s;
+    cudaEvent_t a = nullptr, b = nullptr;
+    Prof(emtk_ctx *c_, int kind_, cudaStream_t s_) : c(c_), kind(kind_), s(s_) {
+        c->stats.launches++;
+        c->stats.kernel_launches[kind]++;
+        if (!c->opt.profile) return;
+        if (cudaEventCreate(&a) != cudaSuccess || cudaEventCreate(&b) != cudaSuccess) {
+            if (a) cudaEventDestroy(a);
+            a = b = nullptr;
+            return;
+        }
+        cudaEventRecord(a, s);
+    }
+    ~Prof() {
+        if (!a) return;
+        cudaEventRecord(b, s);
+        c->pending.push_back({kind, a, b});
+    }
+};
+
+void drain_events(emtk_ctx *c) {
+    for (auto &p : c->pending) {
+        float ms = 0.f;
+        if (cudaEventSynchronize(p.stop) == cudaSuccess && cudaEventElapsedTime(&ms, p.start, p.stop) == cudaSuccess)
+            c->stats.kernel_ms[p.kind] += ms;
+        cudaEventDestroy(p.start);
+        cudaEventDestroy(p.stop);
+    }
+    c->pending.clear();
+}
+
+void count_launch(emtk_ctx *c, int n) {
+    static const int edges[7] = {256, 1024, 2048, 4096, 8192, 16384, 65536};
+    int b = 0;
+    while (b < 7 && n >= edges[b]) ++b;
+    c->stats.batch_hist[b]++;
+    c->stats.chunks++;
+}
+
+// Interval-image workspace large enough for the requests of one table.
+emtk_status ensure_dimg(emtk_ctx *c, size_t bytes, cudaStream_t s) {
+    if (bytes <= c->ws.dimg_bytes) return EMTK_OK;
+    // earlier work on this stream may still read the old buffer
+    cudaError_t e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_status(e);
+    if (c->ws.dimg) cudaFree(c->ws.dimg);
+    c->ws.dimg = nullptr;
+    c->ws.dimg_bytes = 0;
+    const size_t want = bytes + bytes / 4;
+    e = cudaMalloc(&c->ws.dimg, want);
+    if (e != cudaSuccess) return cuda_status(e);
+    c->ws.dimg_bytes = want;
+    return EMTK_OK;
+}
+
+// Network on `n` patches already in the workspace format -> scores via dest.
+emtk_status run_network(emtk_ctx *c, const void *patches, int32_t n, float *const *dest, cudaStream_t s) {
+    if (n <= 0) return EMTK_OK;
+    const int n_pad = n_pad_of(n);
+    const int max_splits = (int)std::max<int64_t>(1, kPartialCap / ((int64_t)n_pad * kN1));
+    cudaError_t e;
+    int splits;
+    if (tensor_precision(c->opt.precision)) {
+        splits = choose_splits_tc(n, c->sm_count, max_splits);
+        Prof prof(c, EMTK_KERNEL_NETWORK, s);
+        e = launch_cnn_tc(c->w, patches, c->opt.precision == EMTK_FP16, n, splits, c->ws.partials, n_pad,
+                          c->ws.status, c->opt.wait_timeout_ns, c->opt.debug_stall, s);
+    } else {
+        splits = choose_splits_fp32(n, c->sm_count, max_splits);
+        Prof prof(c, EMTK_KERNEL_NETWORK, s);
+        e = launch_cnn_fp32(c->w, static_cast<const float *>(patches), n, splits, c->ws.partials, n_pad, s);
+    }
+    if (e != cudaSuccess) return cuda_status(e);
+    {
+        Prof prof(c, EMTK_KERNEL_HEAD, s);
+        e = launch_head(c->w, c->ws.partials, splits, n_pad, n, dest, c->opt.debug_logits, s);
+    }
+    count_launch(c, n);
+    return cuda_status(e);
+}
+
+// Fills a table from requests [r0, r1); returns total hits and image bytes.
+void build_table(const emtk_ctx *c, const emtk_request *reqs, int r0, int r1, emtk_patch_format fmt, ReqTable &t,
+                 int64_t &hits, size_t &img_bytes) {
+    std::memset(&t, 0, sizeof(t));
+    t.n = r1 - r0;
+    hits = 0;
+    int64_t elems = 0;
+    for (int i = 0; i < t.n; ++i) {
+        const emtk_request &q = reqs[r0 + i];
+        ReqDesc &d = t.r[i];
+        d.adc = q.d_adc;
+        d.hits = q.d_hits;
+        d.scores = q.d_scores;
+        d.ld = q.ld;
+        d.nwires = q.nwires;
+        d.nticks = q.nticks;
+        d.nhits = q.nhits;
+        d.nint = q.nticks / kDs;
+        d.pitch = (d.nint + 7) / 8 * 8;
+        d.hit_begin = hits;
+        d.d_off = elems;
+        hits += q.nhits;
+        elems += (int64_t)d.nwires * d.pitch;
+    }
+    img_bytes = (size_t)elems * patch_elem_bytes(fmt);
+    (void)c;
+}
+
+emtk_status run_requests(emtk_ctx *c, const emtk_request *reqs, int32_t nreq, cudaStream_t s) {
+    const emtk_patch_format fmt = patch_format(c->opt.precision);
+    ReqTable *t = new (std::nothrow) ReqTable;
+    if (!t) return EMTK_ERR_OOM;
+    emtk_status st = EMTK_OK;
+    for (int r0 = 0; r0 < nreq && st == EMTK_OK; r0 += kMaxReqPerLaunch) {
+        const int r1 = std::min<int>(nreq, r0 + kMaxReqPerLaunch);
+        int64_t hits;
+        size_t img_bytes;
+        build_table(c, reqs, r0, r1, fmt, *t, hits, img_bytes);
+        if (hits == 0) continue;
+        // planes of requests without hits need no interval image
+        for (int i = 0; i < t->n; ++i)
+            if (t->r[i].nhits == 0) t->r[i].nwires = 0;
+        st = ensure_dimg(c, img_bytes, s);
+        if (st != EMTK_OK) break;
+        cudaError_t e;
+        {
+            Prof prof(c, EMTK_KERNEL_INTERVALS, s);
+            e = launch_interval_images(*t, c->ws.dimg, fmt, s);
+        }
+        if (e != cudaSuccess) {
+            st = cuda_status(e);
+            break;
+        }
+        for (int64_t g0 = 0; g0 < hits && st == EMTK_OK; g0 += c->max_hits) {
+            const int32_t cnt = (int32_t)std::min<int64_t>(c->max_hits, hits - g0);
+            {
+                Prof prof(c, EMTK_KERNEL_GATHER, s);
+                e = launch_gather(*t, c->ws.dimg, fmt, g0, cnt, c->ws.patches, c->ws.dest, out_stride(c), s);
+            }
+            if (e != cudaSuccess) {
+                st = cuda_status(e);
+                break;
+            }
+            st = run_network(c, c->ws.patches, cnt, c->ws.dest, s);
+        }
+        c->stats.hits += hits;
+    }
+    delete t;
+    return st;
+}
+
+}  // namespace
+
+extern "C" {
+
+void emtk_default_options(emtk_options *o) {
+    if (!o) return;
+    o->precision = EMTK_BF16;
+    o->max_hits = 65536;
+    o->debug_logits = 0;
+    o->wait_timeout_ns = 2000000000ll;
+    o->debug_stall = 0;
+    o->profile = 0;
+}
+
+const char *emtk_status_string(emtk_status s) {
+    switch (s) {
+        case EMTK_OK: return "ok";
+        case EMTK_ERR_ARG: return "invalid argument";
+        case EMTK_ERR_ALIGN: return "misaligned buffer or leading dimension";
+        case EMTK_ERR_OOM: return "device allocation failed";
+        case EMTK_ERR_CUDA: return "CUDA error";
+        case EMTK_ERR_TIMEOUT: return "a device-side wait gave up";
+        case EMTK_ERR_UNSUPPORTED: return "unsupported precision or device";
+    }
+    return "unknown status";
+}
+
+emtk_status emtk_create(const emtk_weights *w, const emtk_options *opt, int device, emtk_ctx **out) {
+    if (out) *out = nullptr;
+    if (!w || !out || device < 0) return EMTK_ERR_ARG;
+    const float *all[10] = {w->conv_w, w->conv_b, w->fc1_w, w->fc1_b, w->fc2_w,
+                            w->fc2_b,  w->cls_w,  w->cls_b, w->mic_w, w->mic_b};
+    for (const float *p : all)
+        if (!p) return EMTK_ERR_ARG;
+    emtk_options o;
+    emtk_default_options(&o);
+    if (opt) o = *opt;
+    if (o.precision != EMTK_FP32 && o.precision != EMTK_TF32 && o.precision != EMTK_BF16 &&
+        o.precision != EMTK_FP16)
+        return EMTK_ERR_ARG;
+    if (o.max_hits <= 0 || o.wait_timeout_ns <= 0 || (o.debug_logits != 0 && o.debug_logits != 1) ||
+        (o.profile != 0 && o.profile != 1) || (o.debug_stall != 0 && o.debug_stall != 1))
+        return EMTK_ERR_ARG;
+    if (o.precision == EMTK_TF32) return EMTK_ERR_UNSUPPORTED;
+
+    int ndev = 0;
+    if (cudaGetDeviceCount(&ndev) != cudaSuccess || device >= ndev) return EMTK_ERR_CUDA;
+    DeviceGuard g(device);
+    if (!g.ok) return EMTK_ERR_CUDA;
+    cudaDeviceProp prop;
+    if (cudaGetDeviceProperties(&prop, device) != cudaSuccess) return EMTK_ERR_CUDA;
+    if (!(prop.major == 10 && prop.minor == 3)) return EMTK_ERR_UNSUPPORTED;  // built for sm_103a only
+
+    emtk_ctx *c = new (std::nothrow) emtk_ctx;
+    if (!c) return EMTK_ERR_OOM;
+    c->device = device;
+    c->opt = o;
+    c->max_hits = o.max_hits;
+    c->sm_count = prop.multiProcessorCount;
+    const emtk_patch_format fmt = patch_format(o.precision);
+    cudaError_t e = cudaSuccess;
+    DeviceWeights &d = c->w;
+    if (e == cudaSuccess) e = upload(&d.conv_w, w->conv_w, (size_t)kK * kK * kF);
+    if (e == cudaSuccess) e = upload(&d.conv_b, w->conv_b, kF);
+    if (e == cudaSuccess) e = upload(&d.fc1_b, w->fc1_b, kN1);
+    if (e == cudaSuccess) e = upload(&d.fc2_w, w->fc2_w, (size_t)kN1 * kN2);
+    if (e == cudaSuccess) e = upload(&d.fc2_b, w->fc2_b, kN2);
+    if (e == cudaSuccess) e = upload(&d.cls_w, w->cls_w, (size_t)kN2 * kNC);
+    if (e == cudaSuccess) e = upload(&d.cls_b, w->cls_b, kNC);
+    if (e == cudaSuccess) e = upload(&d.mic_w, w->mic_w, kN2);
+    if (e == cudaSuccess) e = upload(&d.mic_b, w->mic_b, 1);
+    if (e == cudaSuccess) {
+        if (tensor_precision(o.precision)) {
+            e = prepare_tc_weights(d, *w, o.precision == EMTK_FP16);
+            if (e == cudaSuccess) e = init_tc_kernel_attrs();
+        } else {
+            e = upload(&d.fc1_w, w->fc1_w, (size_t)kFc1In * kN1);
+            if (e == cudaSuccess) e = init_fp32_kernel_attrs();
+        }
+    }
+    if (e == cudaSuccess) e = dmalloc(&c->ws.patches, (size_t)o.max_hits * kPatchElems * patch_elem_bytes(fmt));
+    if (e == cudaSuccess) e = dmalloc(&c->ws.dest, (size_t)o.max_hits * sizeof(float *));
+    if (e == cudaSuccess) {
+        c->ws.partial_elems = (size_t)std::max<int64_t>(kPartialCap, (int64_t)n_pad_of(o.max_hits) * kN1);
+        e = dmalloc(&c->ws.partials, c->ws.partial_elems * sizeof(float));
+    }
+    if (e == cudaSuccess) e = dmalloc(&c->ws.status, sizeof(int));
+    if (e == cudaSuccess) e = cudaMemset(c->ws.status, 0, sizeof(int));
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) {
+        free_ctx(c);
+        return cuda_status(e);
+    }
+    *out = c;
+    return EMTK_OK;
+}
+
+emtk_status emtk_destroy(emtk_ctx *c) {
+    if (!c) return EMTK_OK;
+    DeviceGuard g(c->device);
+    cudaDeviceSynchronize();
+    free_ctx(c);
+    return EMTK_OK;
+}
+
+emtk_status emtk_infer_batch(emtk_ctx *c, const emtk_request *reqs, int32_t nreq, emtk_stream stream) {
+    if (!c || nreq < 0 || (nreq > 0 && !reqs)) return EMTK_ERR_ARG;
+    for (int i = 0; i < nreq; ++i) {
+        const emtk_request &q = reqs[i];
+        emtk_status st = check_plane(q.d_adc, q.nwires, q.nticks, q.ld, q.d_hits, q.nhits);
+        if (st != EMTK_OK) return st;
+        if (q.nhits > 0 && q.d_scores == nullptr) return EMTK_ERR_ARG;
+        if ((reinterpret_cast<uintptr_t>(q.d_scores) & 3u) != 0) return EMTK_ERR_ALIGN;
+    }
+    c->stats.calls++;
+    DeviceGuard g(c->device);
+    if (!g.ok) return EMTK_ERR_CUDA;
+    return run_requests(c, reqs, nreq, reinterpret_cast<cudaStream_t>(stream));
+}
+
+emtk_status emtk_infer(emtk_ctx *c, const float *d_adc, int32_t nwires, int32_t nticks, int64_t ld,
+                       const emtk_hit *d_hits, int32_t nhits, float *d_scores, emtk_stream stream) {
+    if (!c) return EMTK_ERR_ARG;
+    emtk_request q{d_adc, nwires, nticks, ld, d_hits, nhits, d_scores};
+    return emtk_infer_batch(c, &q, 1, stream);
+}
+
+emtk_status emtk_extract_patches(emtk_ctx *c, const float *d_adc, int32_t nwires, int32_t nticks, int64_t ld,
+                                 const emtk_hit *d_hits, int32_t nhits, void *d_patches, emtk_patch_format fmt,
+                                 emtk_stream stream) {
+    if (!c) return EMTK_ERR_ARG;
+    if (fmt != EMTK_PATCH_F32 && fmt != EMTK_PATCH_BF16 && fmt != EMTK_PATCH_F16) return EMTK_ERR_ARG;
+    emtk_status st = check_plane(d_adc, nwires, nticks, ld, d_hits, nhits);
+    if (st != EMTK_OK) return st;
+    if (nhits == 0) return EMTK_OK;
+    if (!d_patches) return EMTK_ERR_ARG;
+    if (!aligned16(d_patches)) return EMTK_ERR_ALIGN;
+    DeviceGuard g(c->device);
+    if (!g.ok) return EMTK_ERR_CUDA;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    emtk_request q{d_adc, nwires, nticks, ld, d_hits, nhits, nullptr};
+    ReqTable *t = new (std::nothrow) ReqTable;
+    if (!t) return EMTK_ERR_OOM;
+    int64_t hits;
+    size_t img_bytes;
+    build_table(c, &q, 0, 1, fmt, *t, hits, img_bytes);
+    st = ensure_dimg(c, img_bytes, s);
+    if (st == EMTK_OK) {
+        Prof prof(c, EMTK_KERNEL_INTERVALS, s);
+        st = cuda_status(launch_interval_images(*t, c->ws.dimg, fmt, s));
+    }
+    if (st == EMTK_OK) {
+        Prof prof(c, EMTK_KERNEL_GATHER, s);
+        st = cuda_status(launch_gather(*t, c->ws.dimg, fmt, 0, nhits, d_patches, nullptr, 0, s));
+    }
+    c->stats.calls++;
+    delete t;
+    return st;
+}
+
+emtk_status emtk_infer_patches(emtk_ctx *c, const float *d_patches, int32_t n, float *d_scores,
+                               emtk_stream stream) {
+    if (!c || n < 0) return EMTK_ERR_ARG;
+    if (n == 0) return EMTK_OK;
+    if (!d_patches || !d_scores) return EMTK_ERR_ARG;
+    if (!aligned16(d_patches) || (reinterpret_cast<uintptr_t>(d_scores) & 3u) != 0) return EMTK_ERR_ALIGN;
+    DeviceGuard g(c->device);
+    if (!g.ok) return EMTK_ERR_CUDA;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    const emtk_patch_format fmt = patch_format(c->opt.precision);
+    emtk_status st = EMTK_OK;
+    for (int64_t h0 = 0; h0 < n && st == EMTK_OK; h0 += c->max_hits) {
+        const int32_t cnt = (int32_t)std::min<int64_t>(c->max_hits, n - h0);
+        const float *src = d_patches + h0 * kPatchElems;
+        const void *net_in = src;
+        if (fmt != EMTK_PATCH_F32) {
+            Prof prof(c, EMTK_KERNEL_CONVERT, s);
+            st = cuda_status(launch_convert_patches(src, c->ws.patches, fmt, (int64_t)cnt * kPatchElems, s));
+            net_in = c->ws.patches;
+        }
+        if (st == EMTK_OK) {
+            Prof prof(c, EMTK_KERNEL_CONVERT, s);
+            st = cuda_status(launch_fill_dest(d_scores + h0 * out_stride(c), out_stride(c), c->ws.dest, cnt, s));
+        }
+        if (st == EMTK_OK) st = run_network(c, net_in, cnt, c->ws.dest, s);
+    }
+    c->stats.calls++;
+    c->stats.hits += (uint64_t)n;
+    return st;
+}
+
+emtk_status emtk_check(emtk_ctx *c, emtk_stream stream) {
+    if (!c) return EMTK_ERR_ARG;
+    DeviceGuard g(c->device);
+    if (!g.ok) return EMTK_ERR_CUDA;
+    cudaError_t e = cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return EMTK_ERR_CUDA;
+    int status = 0;
+    e = cudaMemcpy(&status, c->ws.status, sizeof(int), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return EMTK_ERR_CUDA;
+    if (status != 0) {
+        e = cudaMemset(c->ws.status, 0, sizeof(int));
+        if (e != cudaSuccess) return EMTK_ERR_CUDA;
+        return EMTK_ERR_TIMEOUT;
+    }
+    return EMTK_OK;
+}
+
+emtk_status emtk_get_stats(emtk_ctx *c, emtk_stats *out) {
+    if (!c || !out) return EMTK_ERR_ARG;
+    if (!c->pending.empty()) {
+        DeviceGuard g(c->device);
+        drain_events(c);
+    }
+    *out = c->stats;
+    return EMTK_OK;
+}
+
+}  // extern "C"

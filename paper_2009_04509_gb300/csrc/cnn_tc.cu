@@ -1,0 +1,614 @@
+// 16-bit network path on the sm_103a tensor cores (EMTK_BF16 / EMTK_FP16):
+// the conv 5x5x48 + ReLU (Sec. 2.2) fused into dense-1 (92,928 -> 128), so
+// the 92,928 conv activations of a hit never leave the SM.
+//
+// One CTA = 128 hits (one TMEM lane each) x one segment of the dense-1 input
+// dimension, walked conv position by conv position (p = y*44 + x; the
+// dense-1 input index is p*48 + c, the paper's channels-last flatten).
+// Per position:
+//   builder warps   write the hit's 5x5 im2col row (25 taps, two bias taps
+//                   of 1.0, zero padding to K = 32) into TMEM;
+//   MMA thread      conv MMA  D[128 x 48] = A_tmem[128 x 32] * Bconv[32 x 48]
+//                   (the conv bias rides on the two constant taps);
+//   epilogue warps  ReLU + round the conv tile to 16 bit, written back into
+//                   TMEM over the conv accumulator;
+//   MMA thread      dense-1 MMA  ACC[128 x 128] += A_tmem[128 x 48] * W1[48 x 128]
+//                   with W1 streamed through a 4-deep TMA ring in shared
+//                   memory (128-byte swizzle, 4 positions per stage).
+// Both MMAs take their A operand from tensor memory; shared memory only
+// carries the W1 stream and the conv weights.  Every wait is bounded: on
+// timeout the CTA raises an abort flag, sets bit 0 of the status word, waits
+// for its in-flight copies and MMAs, frees TMEM and returns.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cudaTypedefs.h>
+
+#include <vector>
+
+#include "emtk_internal.h"
+
+namespace emtk {
+namespace {
+
+constexpr int kThreadsTC = 320;  // warp 0 TMA, warp 1 MMA, warps 2-5 builder, warps 6-9 epilogue
+constexpr int kStages = 6;       // TMEM stages, one conv position each
+constexpr int kW1Stages = 4;     // shared-memory stages of W1
+constexpr int kPosPerW1 = 4;     // conv positions per W1 stage
+constexpr int kW1Steps = kPos / kPosPerW1;                  // 484
+constexpr int kW1Box = 64;                                   // K elements per TMA box (128 B)
+constexpr int kW1BoxBytes = kW1Box * kN1 * 2;                // 16384
+constexpr int kBoxesPerStage = kPosPerW1 * kF / kW1Box;      // 3
+constexpr int kW1StageBytes = kBoxesPerStage * kW1BoxBytes;  // 49152
+constexpr int kKBlocks = kFc1In / kW1Box;                    // 1452
+constexpr int kConvK = 32;                                   // 25 taps + 2 bias taps + 5 zeros
+constexpr int kConvBBytes = kF * 128;                        // 48 rows of one 128-byte swizzle span
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kAccCol = 0;
+constexpr uint32_t kStageCol0 = 128;
+constexpr uint32_t kStageCols = 64;
+constexpr uint32_t kIm2colOff = 48;
+constexpr int kLag = 2;          // dense-1 of position p is issued after the conv of p + 2
+
+constexpr int kOffW1 = 0;
+constexpr int kOffConvB = kOffW1 + kW1Stages * kW1StageBytes;
+constexpr int kOffBar = kOffConvB + kConvBBytes;
+// barrier indices
+constexpr int kBarW1Full = 0;
+constexpr int kBarW1Empty = kBarW1Full + kW1Stages;
+constexpr int kBarIm2col = kBarW1Empty + kW1Stages;
+constexpr int kBarConv = kBarIm2col + kStages;
+constexpr int kBarAct = kBarConv + kStages;
+constexpr int kBarFree = kBarAct + kStages;
+constexpr int kBarAcc = kBarFree + kStages;
+constexpr int kBarStall = kBarAcc + 1;
+constexpr int kBarDrain = kBarStall + 1;
+constexpr int kNumBars = kBarDrain + 1;
+constexpr int kOffTmemSlot = kOffBar + kNumBars * 8;
+constexpr int kOffAbort = kOffTmemSlot + 4;
+constexpr int kSmemUsed = kOffAbort + 4;
+constexpr int kSmemBytesTC = kSmemUsed + 1024;  // slack for 1024-byte alignment
+static_assert(kSmemBytesTC <= 232448, "shared memory budget");
+static_assert(kStageCol0 + kStages * kStageCols <= kTmemCols, "TMEM budget");
+
+// ------------------------------------------------------------ PTX helpers
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ uint64_t global_timer_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+struct Guard {
+    volatile uint32_t *abort;
+    int *status;
+    int64_t timeout_ns;
+};
+
+// Waits for the phase of `parity` to complete.  Gives up (false) when the
+// CTA's abort flag is raised or after timeout_ns, raising the flag and the
+// status bit itself in the second case.
+__device__ __noinline__ bool wait_bounded(uint32_t bar, uint32_t parity, Guard g) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = global_timer_ns();
+    for (uint32_t i = 1;; ++i) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if ((i & 31u) == 0) {
+            if (*g.abort) return false;
+            if ((int64_t)(global_timer_ns() - t0) > g.timeout_ns) {
+                *g.abort = 1u;
+                atomicOr(g.status, 1);
+                return false;
+            }
+        }
+    }
+}
+
+// Lane 0 waits; the outcome is broadcast so the whole warp takes the same path.
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, Guard g, int lane) {
+    int ok = 1;
+    if (lane == 0) ok = wait_bounded(bar, parity, g) ? 1 : 0;
+    ok = __shfl_sync(0xffffffffu, ok, 0);
+    __syncwarp();
+    return ok != 0;
+}
+
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int c0, int c1,
+                                            int c2) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4, %5}], "
+        "[%2];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "r"(c2)
+        : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// D[tmem] (+)= A[tmem] * B[smem desc], kind::f16, one CTA.
+__device__ __forceinline__ void mma_ts(uint32_t d, uint32_t a, uint64_t bdesc, uint32_t idesc, uint32_t accum) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d),
+        "r"(a), "l"(bdesc), "r"(idesc), "r"(accum)
+        : "memory");
+}
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+                 : "memory");
+}
+
+#define EMTK_R16(r, o)                                                                                       \
+    "=r"(r[o + 0]), "=r"(r[o + 1]), "=r"(r[o + 2]), "=r"(r[o + 3]), "=r"(r[o + 4]), "=r"(r[o + 5]),         \
+        "=r"(r[o + 6]), "=r"(r[o + 7]), "=r"(r[o + 8]), "=r"(r[o + 9]), "=r"(r[o + 10]), "=r"(r[o + 11]), \
+        "=r"(r[o + 12]), "=r"(r[o + 13]), "=r"(r[o + 14]), "=r"(r[o + 15])
+
+template <int O, int N>
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[N]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : EMTK_R16(r, O)
+        : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+__device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
+template <int O, int N>
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[N]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
+            taddr),
+        "r"(r[O + 0]), "r"(r[O + 1]), "r"(r[O + 2]), "r"(r[O + 3]), "r"(r[O + 4]), "r"(r[O + 5]), "r"(r[O + 6]),
+        "r"(r[O + 7]), "r"(r[O + 8]), "r"(r[O + 9]), "r"(r[O + 10]), "r"(r[O + 11]), "r"(r[O + 12]), "r"(r[O + 13]),
+        "r"(r[O + 14]), "r"(r[O + 15])
+        : "memory");
+}
+template <int O, int N>
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&r)[N]) {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr), "r"(r[O + 0]),
+                 "r"(r[O + 1]), "r"(r[O + 2]), "r"(r[O + 3]), "r"(r[O + 4]), "r"(r[O + 5]), "r"(r[O + 6]),
+                 "r"(r[O + 7])
+                 : "memory");
+}
+// Makes later uses of r depend on the preceding tcgen05.wait::ld.
+template <int N>
+__device__ __forceinline__ void reg_fence(uint32_t (&r)[N]) {
+#pragma unroll
+    for (int i = 0; i < N; ++i) asm volatile("" : "+r"(r[i]));
+}
+
+template <bool FP16>
+__device__ __forceinline__ uint32_t relu_pack(uint32_t lo, uint32_t hi) {
+    uint32_t d;
+    if (FP16)
+        asm("cvt.rn.relu.f16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(__uint_as_float(hi)), "f"(__uint_as_float(lo)));
+    else
+        asm("cvt.rn.relu.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(__uint_as_float(hi)), "f"(__uint_as_float(lo)));
+    return d;
+}
+
+// Instruction descriptor, kind::f16: fp32 accumulate, both operands K-major.
+__host__ __device__ constexpr uint32_t make_idesc(int M, int N, bool fp16) {
+    return (1u << 4) | ((fp16 ? 0u : 1u) << 7) | ((fp16 ? 0u : 1u) << 10) | ((uint32_t)(N >> 3) << 17) |
+           ((uint32_t)(M >> 4) << 24);
+}
+
+// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups
+// 1024 bytes apart (SBO), sm_100 descriptor version.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
+           ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+
+// ------------------------------------------------------------------ kernel
+template <bool FP16>
+__global__ void __launch_bounds__(kThreadsTC, 1)
+    cnn_tc_kernel(const __grid_constant__ CUtensorMap tmap_w1, const uint16_t *__restrict__ patches, int n,
+                  const uint16_t *__restrict__ convB_g, float *__restrict__ partials, int n_pad, int splits,
+                  int *status, long long timeout_ns, int debug_stall) {
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw_u32 = smem_u32(smem_raw);
+    const uint32_t base = (raw_u32 + 1023u) & ~1023u;
+    uint8_t *gbase = smem_raw + (base - raw_u32);
+    const uint32_t sW1 = base + kOffW1;
+    const uint32_t sConvB = base + kOffConvB;
+    auto bar = [&](int i) -> uint32_t { return base + kOffBar + 8u * (uint32_t)i; };
+    volatile uint32_t *tmem_slot = reinterpret_cast<volatile uint32_t *>(gbase + kOffTmemSlot);
+    volatile uint32_t *abort_flag = reinterpret_cast<volatile uint32_t *>(gbase + kOffAbort);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int m_tile = blockIdx.x;
+    const int seg = blockIdx.y;
+    const int j0 = (int)((int64_t)seg * kW1Steps / splits);
+    const int j1 = (int)((int64_t)(seg + 1) * kW1Steps / splits);
+    const int nW1 = j1 - j0;
+    const int p0 = j0 * kPosPerW1;
+    const int p1 = j1 * kPosPerW1;
+    const int npos = p1 - p0;
+    const Guard guard{abort_flag, status, (int64_t)timeout_ns};
+
+    // ---- set-up: conv B operand into swizzled smem, barriers, TMEM
+    for (int idx = threadIdx.x; idx < kF * 8; idx += kThreadsTC) {
+        const int row = idx >> 3, chunk = idx & 7;
+        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+        if (chunk < kConvK / 8) v = __ldg(reinterpret_cast<const uint4 *>(convB_g + row * kConvK) + chunk);
+        *reinterpret_cast<uint4 *>(gbase + kOffConvB + row * 128 + ((chunk ^ (row & 7)) << 4)) = v;
+    }
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < kW1Stages; ++i) {
+            mbar_init(bar(kBarW1Full + i), 1);
+            mbar_init(bar(kBarW1Empty + i), 1);
+        }
+        for (int i = 0; i < kStages; ++i) {
+            mbar_init(bar(kBarIm2col + i), 4);
+            mbar_init(bar(kBarConv + i), 1);
+            mbar_init(bar(kBarAct + i), 4);
+            mbar_init(bar(kBarFree + i), 1);
+        }
+        mbar_init(bar(kBarAcc), 1);
+        mbar_init(bar(kBarStall), 1);
+        mbar_init(bar(kBarDrain), 1);
+        *abort_flag = 0u;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(base + kOffTmemSlot),
+                     "r"(kTmemCols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0) {
+        // ================================================= TMA producer (W1)
+        if (lane == 0) {
+            int issued = 0;
+            bool ok = true;
+            for (int jj = 0; jj < nW1; ++jj) {
+                const int wj = jj % kW1Stages;
+                const uint32_t use = (uint32_t)(jj / kW1Stages);
+                if (jj >= kW1Stages && !wait_bounded(bar(kBarW1Empty + wj), (use - 1u) & 1u, guard)) {
+                    ok = false;
+                    break;
+                }
+                if (*abort_flag) {
+                    ok = false;
+                    break;
+                }
+                mbar_expect_tx(bar(kBarW1Full + wj), kW1StageBytes);
+#pragma unroll
+                for (int a = 0; a < kBoxesPerStage; ++a)
+                    tma_load_3d(sW1 + wj * kW1StageBytes + a * kW1BoxBytes, &tmap_w1, bar(kBarW1Full + wj), 0, 0,
+                                kBoxesPerStage * (j0 + jj) + a);
+                ++issued;
+            }
+            if (!ok) {  // let copies in flight land before the CTA's memory goes away
+                for (int jj = issued > kW1Stages ? issued - kW1Stages : 0; jj < issued; ++jj) {
+                    const uint32_t b = bar(kBarW1Full + jj % kW1Stages);
+                    const uint32_t par = (uint32_t)(jj / kW1Stages) & 1u;
+                    const uint64_t t0 = global_timer_ns();
+                    while (!mbar_try_wait(b, par) && (int64_t)(global_timer_ns() - t0) < (int64_t)timeout_ns) {
+                    }
+                }
+            }
+        }
+    } else if (warp == 1) {
+        // ======================================================= MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t idesc_conv = make_idesc(128, kF, FP16);
+            constexpr uint32_t idesc_fc1 = make_idesc(128, kN1, FP16);
+            const uint64_t convb_desc = sw128_desc(sConvB);
+            bool ok = true;
+            if (debug_stall) ok = wait_bounded(bar(kBarStall), 0u, guard);  // nothing arrives here
+            for (int k = 0; ok && k < npos + kLag; ++k) {
+                if (k < npos) {
+                    const int s = k % kStages;
+                    const uint32_t use = (uint32_t)(k / kStages);
+                    if (!wait_bounded(bar(kBarIm2col + s), use & 1u, guard)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t d = tmem + kStageCol0 + (uint32_t)s * kStageCols;
+                    mma_ts(d, d + kIm2colOff, convb_desc, idesc_conv, 0u);
+                    mma_ts(d, d + kIm2colOff + 8u, convb_desc + (32u >> 4), idesc_conv, 1u);
+                    mma_commit(bar(kBarConv + s));
+                }
+                const int qq = k - kLag;
+                if (qq >= 0) {
+                    const int sq = qq % kStages;
+                    const uint32_t uq = (uint32_t)(qq / kStages);
+                    const int jj = qq / kPosPerW1;
+                    const int wj = jj % kW1Stages;
+                    const int pin = qq % kPosPerW1;
+                    if (pin == 0 && !wait_bounded(bar(kBarW1Full + wj), (uint32_t)(jj / kW1Stages) & 1u, guard)) {
+                        ok = false;
+                        break;
+                    }
+                    if (!wait_bounded(bar(kBarAct + sq), uq & 1u, guard)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint64_t wdesc = sw128_desc(sW1 + wj * kW1StageBytes);
+                    const uint32_t a = tmem + kStageCol0 + (uint32_t)sq * kStageCols;
+#pragma unroll
+                    for (int t = 0; t < 3; ++t) {
+                        const int step = pin * 3 + t;
+                        const uint64_t bd = wdesc + (uint64_t)(((step >> 2) * kW1BoxBytes + (step & 3) * 32) >> 4);
+                        mma_ts(tmem + kAccCol, a + 8u * t, bd, idesc_fc1, (qq > 0 || t > 0) ? 1u : 0u);
+                    }
+                    mma_commit(bar(kBarFree + sq));
+                    if (pin == kPosPerW1 - 1) mma_commit(bar(kBarW1Empty + wj));
+                }
+            }
+            if (ok) mma_commit(bar(kBarAcc));
+            // every MMA issued so far completes before TMEM is released
+            mma_commit(bar(kBarDrain));
+            const uint64_t t0 = global_timer_ns();
+            while (!mbar_try_wait(bar(kBarDrain), 0u) && (int64_t)(global_timer_ns() - t0) < (int64_t)timeout_ns) {
+            }
+        }
+    } else if (warp < 6) {
+        // ================================================ im2col builder
+        const int q = warp & 3;
+        const int row = 32 * q + lane;
+        const int64_t hit = (int64_t)m_tile * 128 + row;
+        const bool valid = hit < n;
+        const uint4 *prow = reinterpret_cast<const uint4 *>(patches) + (valid ? hit : 0) * (kPatchElems / 8);
+        const uint32_t one = FP16 ? 0x3C00u : 0x3F80u;
+        const uint32_t lane_tmem = tmem + ((uint32_t)(32 * q) << 16);
+        const int y_first = p0 / kQ;
+        const int y_last = (p1 - 1) / kQ;
+        bool ok = npos > 0;
+        for (int y = y_first; ok && y <= y_last; ++y) {
+            uint32_t R[kK][24];
+#pragma unroll
+            for (int i = 0; i < kK; ++i) {
+#pragma unroll
+                for (int u = 0; u < 6; ++u) {
+                    const uint4 v = valid ? __ldg(prow + (y + i) * 6 + u) : make_uint4(0u, 0u, 0u, 0u);
+                    R[i][4 * u + 0] = v.x;
+                    R[i][4 * u + 1] = v.y;
+                    R[i][4 * u + 2] = v.z;
+                    R[i][4 * u + 3] = v.w;
+                }
+            }
+#pragma unroll
+            for (int x = 0; x < kQ; ++x) {
+                const int p = y * kQ + x;
+                if (p < p0 || p >= p1) continue;
+                const int k = p - p0;
+                const int s = k % kStages;
+                const uint32_t use = (uint32_t)(k / kStages);
+                if (k >= kStages && !warp_wait(bar(kBarFree + s), (use - 1u) & 1u, guard, lane)) {
+                    ok = false;
+                    break;
+                }
+                uint32_t v[16];
+#pragma unroll
+                for (int pr = 0; pr < 13; ++pr) {
+                    const int t0 = 2 * pr, t1 = 2 * pr + 1;
+                    const int e0 = x + t0 % kK;
+                    const uint32_t sel_lo = (e0 & 1) ? 0x32u : 0x10u;
+                    const uint32_t lo = R[t0 / kK][e0 >> 1];
+                    if (t1 < kK * kK) {
+                        const int e1 = x + t1 % kK;
+                        const uint32_t sel = sel_lo | (((e1 & 1) ? 0x76u : 0x54u) << 8);
+                        v[pr] = __byte_perm(lo, R[t1 / kK][e1 >> 1], sel);
+                    } else {
+                        v[pr] = __byte_perm(lo, one, sel_lo | (0x54u << 8));  // tap 25 = 1.0
+                    }
+                }
+                v[13] = one;  // tap 26 = 1.0, tap 27 = 0
+                v[14] = 0u;
+                v[15] = 0u;
+                tmem_st16<0>(lane_tmem + kStageCol0 + (uint32_t)s * kStageCols + kIm2colOff, v);
+                tmem_st_wait();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar(kBarIm2col + s));
+            }
+        }
+    } else {
+        // ================================== conv epilogue + dense-1 store
+        const int q = warp & 3;
+        const int row = 32 * q + lane;
+        const int64_t hit = (int64_t)m_tile * 128 + row;
+        const uint32_t lane_tmem = tmem + ((uint32_t)(32 * q) << 16);
+        bool ok = true;
+        for (int k = 0; k < npos; ++k) {
+            const int s = k % kStages;
+            if (!warp_wait(bar(kBarConv + s), (uint32_t)(k / kStages) & 1u, guard, lane)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t d = lane_tmem + kStageCol0 + (uint32_t)s * kStageCols;
+            uint32_t f[48];
+            tmem_ld16<0>(d, f);
+            tmem_ld16<16>(d + 16u, f);
+            tmem_ld16<32>(d + 32u, f);
+            tmem_ld_wait();
+            reg_fence(f);
+            uint32_t o[24];
+#pragma unroll
+            for (int i = 0; i < 24; ++i) o[i] = relu_pack<FP16>(f[2 * i], f[2 * i + 1]);
+            tmem_st16<0>(d, o);
+            tmem_st8<16>(d + 16u, o);
+            tmem_st_wait();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(kBarAct + s));
+        }
+        if (ok && npos > 0 && warp_wait(bar(kBarAcc), 0u, guard, lane)) {
+            tc_fence_after();
+            float *dst = partials + ((int64_t)seg * n_pad + hit) * kN1;
+#pragma unroll
+            for (int c = 0; c < kN1 / 32; ++c) {
+                uint32_t r[32];
+                tmem_ld16<0>(lane_tmem + kAccCol + 32u * c, r);
+                tmem_ld16<16>(lane_tmem + kAccCol + 32u * c + 16u, r);
+                tmem_ld_wait();
+                reg_fence(r);
+                if (hit < n) {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e)
+                        reinterpret_cast<float4 *>(dst + 32 * c)[e] =
+                            make_float4(__uint_as_float(r[4 * e]), __uint_as_float(r[4 * e + 1]),
+                                        __uint_as_float(r[4 * e + 2]), __uint_as_float(r[4 * e + 3]));
+                }
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        __syncwarp();
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
+    }
+}
+
+uint16_t to16(float v, bool fp16) {
+    if (fp16) {
+        __half h = __float2half_rn(v);
+        return *reinterpret_cast<uint16_t *>(&h);
+    }
+    __nv_bfloat16 b = __float2bfloat16_rn(v);
+    return *reinterpret_cast<uint16_t *>(&b);
+}
+float from16(uint16_t u, bool fp16) {
+    if (fp16) {
+        __half h;
+        *reinterpret_cast<uint16_t *>(&h) = u;
+        return __half2float(h);
+    }
+    __nv_bfloat16 b;
+    *reinterpret_cast<uint16_t *>(&b) = u;
+    return __bfloat162float(b);
+}
+
+}  // namespace
+
+cudaError_t init_tc_kernel_attrs() {
+    cudaError_t e = cudaFuncSetAttribute(cnn_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         kSmemBytesTC);
+    if (e != cudaSuccess) return e;
+    return cudaFuncSetAttribute(cnn_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytesTC);
+}
+
+cudaError_t prepare_tc_weights(DeviceWeights &w, const emtk_weights &hw, bool fp16) {
+    // dense-1 weights, tiled [K/64][128][64] so that each TMA box is 16 KB of
+    // contiguous memory: tile kb holds W1[kb*64 + kk][nn] at [kb][nn][kk].
+    std::vector<uint16_t> tiles((size_t)kFc1In * kN1);
+    for (int kb = 0; kb < kKBlocks; ++kb)
+        for (int nn = 0; nn < kN1; ++nn)
+            for (int kk = 0; kk < kW1Box; ++kk)
+                tiles[((size_t)kb * kN1 + nn) * kW1Box + kk] = to16(hw.fc1_w[(size_t)(kb * kW1Box + kk) * kN1 + nn], fp16);
+    // conv B operand [48 filters][32]: taps 0..24, bias hi, bias lo, zeros
+    std::vector<uint16_t> cb((size_t)kF * kConvK, 0);
+    for (int f = 0; f < kF; ++f) {
+        for (int t = 0; t < kK * kK; ++t) cb[f * kConvK + t] = to16(hw.conv_w[t * kF + f], fp16);
+        const uint16_t hi = to16(hw.conv_b[f], fp16);
+        cb[f * kConvK + 25] = hi;
+        cb[f * kConvK + 26] = to16(hw.conv_b[f] - from16(hi, fp16), fp16);
+    }
+    cudaError_t e = cudaMalloc(&w.w1_tiles, tiles.size() * 2);
+    if (e != cudaSuccess) return e;
+    e = cudaMemcpy(w.w1_tiles, tiles.data(), tiles.size() * 2, cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return e;
+    e = cudaMalloc(&w.convB, cb.size() * 2);
+    if (e != cudaSuccess) return e;
+    e = cudaMemcpy(w.convB, cb.data(), cb.size() * 2, cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return e;
+
+    void *fn = nullptr;
+    cudaDriverEntryPointQueryResult qr;
+    e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &qr);
+    if (e != cudaSuccess || fn == nullptr || qr != cudaDriverEntryPointSuccess) return cudaErrorNotSupported;
+    auto encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    CUtensorMap *map = new CUtensorMap;
+    cuuint64_t dims[3] = {(cuuint64_t)kW1Box, (cuuint64_t)kN1, (cuuint64_t)kKBlocks};
+    cuuint64_t strides[2] = {(cuuint64_t)kW1Box * 2, (cuuint64_t)kW1Box * kN1 * 2};
+    cuuint32_t box[3] = {(cuuint32_t)kW1Box, (cuuint32_t)kN1, 1u};
+    cuuint32_t estr[3] = {1u, 1u, 1u};
+    CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_UINT16, 3, w.w1_tiles, dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) {
+        delete map;
+        return cudaErrorInvalidValue;
+    }
+    w.w1_tmap = map;
+    return cudaSuccess;
+}
+
+// Splits of the dense-1 input (in W1 stages of 4 positions) so that
+// m_tiles x splits CTAs fill the SMs in few, even waves.  Time model per
+// wave: the segment's stages plus a fixed cost of about 6 stages (pipeline
+// fill and drain, partial-sum store).
+int choose_splits_tc(int n, int sm_count, int max_splits) {
+    const int m_tiles = (n + 127) / 128;
+    int best = 1;
+    double best_t = 1e30;
+    const int cap = max_splits < kW1Steps / 4 ? max_splits : kW1Steps / 4;
+    for (int s = 1; s <= cap; ++s) {
+        const int64_t ctas = (int64_t)m_tiles * s;
+        const int64_t waves = (ctas + sm_count - 1) / sm_count;
+        const double t = (double)waves * ((double)kW1Steps / s + 6.0);
+        if (t < best_t - 1e-9) {
+            best_t = t;
+            best = s;
+        }
+    }
+    return best;
+}
+
+cudaError_t launch_cnn_tc(const DeviceWeights &w, const void *patches, bool fp16, int32_t n, int splits,
+                          float *partials, int n_pad, int *status, int64_t timeout_ns, int debug_stall,
+                          cudaStream_t s) {
+    if (n <= 0) return cudaSuccess;
+    const CUtensorMap &map = *static_cast<const CUtensorMap *>(w.w1_tmap);
+    dim3 grid((n + 127) / 128, splits);
+    if (fp16)
+        cnn_tc_kernel<true><<<grid, kThreadsTC, kSmemBytesTC, s>>>(map, static_cast<const uint16_t *>(patches), n,
+                                                                   w.convB, partials, n_pad, splits, status,
+                                                                   (long long)timeout_ns, debug_stall);
+    else
+        cnn_tc_kernel<false><<<grid, kThreadsTC, kSmemBytesTC, s>>>(map, static_cast<const uint16_t *>(patches), n,
+                                                                    w.convB, partials, n_pad, splits, status,
+                                                                    (long long)timeout_ns, debug_stall);
+    return cudaGetLastError();
+}
+
+}  // namespace emtk

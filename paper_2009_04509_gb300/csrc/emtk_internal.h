@@ -1,0 +1,131 @@
+// Internal declarations shared by the library's translation units.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <vector>
+
+#include "../../include/emtk.h"
+
+namespace emtk {
+
+// Geometry of the method (Sec. 2.1, Sec. 2.2).
+constexpr int kPatch = 48;                           // patch side
+constexpr int kDs = 6;                               // ticks per time interval
+constexpr int kHalf = kPatch / 2;                    // hit sits at row/col 24
+constexpr int kK = 5;                                // conv kernel side
+constexpr int kF = 48;                               // conv filters
+constexpr int kQ = kPatch - kK + 1;                  // 44
+constexpr int kPos = kQ * kQ;                        // 1936 conv positions
+constexpr int kFc1In = kPos * kF;                    // 92,928
+constexpr int kN1 = 128;
+constexpr int kN2 = 32;
+constexpr int kNC = 3;
+constexpr int kPatchElems = kPatch * kPatch;         // 2304
+
+// Requests handled by one extraction launch (kernel-parameter table).
+constexpr int kMaxReqPerLaunch = 64;
+
+struct ReqDesc {
+    const float *adc;
+    const emtk_hit *hits;
+    float *scores;        // output rows of this request
+    int64_t ld;
+    int64_t hit_begin;    // first index of this request in the concatenated hit list
+    int64_t d_off;        // element offset of its interval image in the workspace
+    int32_t nwires;
+    int32_t nticks;
+    int32_t nhits;
+    int32_t nint;         // complete time intervals: nticks / 6
+    int32_t pitch;        // row pitch of the interval image: nint rounded up to 8
+    int32_t pad;
+};
+
+struct ReqTable {
+    int32_t n;
+    int32_t pad;
+    ReqDesc r[kMaxReqPerLaunch];
+};
+
+// Per-context workspace (device).
+struct Workspace {
+    void *dimg = nullptr;        // interval images of the planes of one launch
+    size_t dimg_bytes = 0;
+    void *patches = nullptr;     // [max_hits][48][48] in the precision's patch format
+    float **dest = nullptr;      // [max_hits] output row of each hit
+    float *partials = nullptr;   // [max_splits][max_hits_pad][128]
+    size_t partial_elems = 0;
+    int *status = nullptr;       // device status word (bit 0: a wait gave up)
+};
+
+struct DeviceWeights {
+    float *conv_w = nullptr;     // [25][48] fp32
+    float *conv_b = nullptr;     // [48]
+    float *fc1_w = nullptr;      // [92928][128] fp32 (fp32 path only)
+    float *fc1_b = nullptr;      // [128]
+    float *fc2_w = nullptr;      // [128][32]
+    float *fc2_b = nullptr;
+    float *cls_w = nullptr;      // [32][3]
+    float *cls_b = nullptr;
+    float *mic_w = nullptr;      // [32]
+    float *mic_b = nullptr;
+    uint16_t *w1_tiles = nullptr;  // 16-bit dense-1 weights, tiled for TMA: [1452][128][64]
+    uint16_t *convB = nullptr;     // 16-bit conv B operand: [48][32] (taps 0-24, bias hi, bias lo, zeros)
+    void *w1_tmap = nullptr;       // host copy of the TMA descriptor (CUtensorMap, 128 B)
+};
+
+}  // namespace emtk
+
+struct emtk_pending_event {
+    int kind;
+    cudaEvent_t start, stop;
+};
+
+struct emtk_ctx {
+    int device = 0;
+    std::vector<emtk_pending_event> pending;  // profile mode: launches not yet read back
+    emtk_options opt{};
+    int max_hits = 0;
+    int max_splits = 0;
+    int sm_count = 0;
+    emtk::DeviceWeights w;
+    emtk::Workspace ws;
+    emtk_stats stats{};
+};
+
+namespace emtk {
+
+// ---- kernels launched from the API (each returns cudaGetLastError()).
+// Interval images of every request plane: img[r] is [nwires][nint] of the
+// patch format (fp32 or 16-bit), at element offset r.d_off.
+cudaError_t launch_interval_images(const ReqTable &t, void *dimg, emtk_patch_format fmt, cudaStream_t s);
+// Patches of hits [g0, g0+count) of the concatenated list (global index).
+// Writes patches[(g - g0)] and, if dest != null, dest[g - g0] = output row.
+cudaError_t launch_gather(const ReqTable &t, const void *dimg, emtk_patch_format fmt, int64_t g0,
+                          int32_t count, void *patches, float **dest, int out_stride, cudaStream_t s);
+// Patch cut straight from the planes into caller memory (emtk_extract_patches).
+cudaError_t launch_convert_patches(const float *src, void *dst, emtk_patch_format fmt, int64_t n,
+                                   cudaStream_t s);
+cudaError_t launch_fill_dest(float *scores, int out_stride, float **dest, int32_t n, cudaStream_t s);
+
+// Network: dense-1 partial sums [splits][n_pad][128] from patches.
+cudaError_t launch_cnn_fp32(const DeviceWeights &w, const float *patches, int32_t n, int splits,
+                            float *partials, int n_pad, cudaStream_t s);
+cudaError_t launch_cnn_tc(const DeviceWeights &w, const void *patches, bool fp16, int32_t n,
+                          int splits, float *partials, int n_pad, int *status, int64_t timeout_ns,
+                          int debug_stall, cudaStream_t s);
+// Sum of partials + bias + ReLU, dense-2, heads; scores to dest[h].
+cudaError_t launch_head(const DeviceWeights &w, const float *partials, int splits, int n_pad,
+                        int32_t n, float *const *dest, int debug_logits, cudaStream_t s);
+
+// Kernel attributes (dynamic shared memory), set once per device at create.
+cudaError_t init_fp32_kernel_attrs();
+cudaError_t init_tc_kernel_attrs();
+
+// Host helpers for the tensor-core weights (cnn_tc.cu).
+cudaError_t prepare_tc_weights(DeviceWeights &w, const emtk_weights &hw, bool fp16);
+int choose_splits_tc(int n, int sm_count, int max_splits);
+int choose_splits_fp32(int n, int sm_count, int max_splits);
+
+}  // namespace emtk

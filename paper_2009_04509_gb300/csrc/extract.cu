@@ -1,0 +1,225 @@
+// Patch extraction (Sec. 2.1): every hit gets a 48x48 patch, rows = wires,
+// columns = time intervals of 6 ticks, centred on the hit (row 24 / column
+// 24); pixels outside the plane are zero.
+//
+// Two HBM-friendly passes instead of one gather per hit:
+//   1. interval image: each plane's ticks are reduced once to its interval
+//      values (fp32 sum of the 6 ticks left to right, one fp32 divide by 6),
+//      stored in the patch format.  Reads every plane byte exactly once
+//      (16-byte vector loads, streaming), writes 1/6 of it (stays in L2).
+//   2. gather: each patch is copied out of the L2-resident interval image.
+// Hits of windows that overlap read the same interval values, so the plane
+// is never re-read per hit.
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+
+#include "emtk_internal.h"
+
+namespace emtk {
+namespace {
+
+__device__ __forceinline__ float interval_sum(float a0, float a1, float a2, float a3, float a4, float a5) {
+    // fixed order: ((((a0 + a1) + a2) + a3) + a4) + a5, no contraction possible
+    float s = __fadd_rn(a0, a1);
+    s = __fadd_rn(s, a2);
+    s = __fadd_rn(s, a3);
+    s = __fadd_rn(s, a4);
+    s = __fadd_rn(s, a5);
+    return __fdiv_rn(s, 6.0f);
+}
+
+template <int FMT>
+__device__ __forceinline__ void store2(void *base, int64_t idx, float v0, float v1, bool two) {
+    if (FMT == EMTK_PATCH_F32) {
+        float *p = static_cast<float *>(base) + idx;
+        if (two) {
+            *reinterpret_cast<float2 *>(p) = make_float2(v0, v1);
+        } else {
+            p[0] = v0;
+        }
+    } else if (FMT == EMTK_PATCH_BF16) {
+        __nv_bfloat16 *p = static_cast<__nv_bfloat16 *>(base) + idx;
+        if (two) {
+            __nv_bfloat162 h;
+            h.x = __float2bfloat16_rn(v0);
+            h.y = __float2bfloat16_rn(v1);
+            *reinterpret_cast<__nv_bfloat162 *>(p) = h;
+        } else {
+            p[0] = __float2bfloat16_rn(v0);
+        }
+    } else {
+        __half *p = static_cast<__half *>(base) + idx;
+        if (two) {
+            *reinterpret_cast<__half2 *>(p) = __halves2half2(__float2half_rn(v0), __float2half_rn(v1));
+        } else {
+            p[0] = __float2half_rn(v0);
+        }
+    }
+}
+
+// One thread = two consecutive intervals of one wire (12 ticks = 48 bytes,
+// 16-byte aligned because ld % 4 == 0 and the plane is 16-byte aligned).
+// grid.y = request; image rows have an even pitch and start at an even
+// element offset, so the pair store is aligned too.
+template <int FMT>
+__global__ void __launch_bounds__(256) interval_image_kernel(const __grid_constant__ ReqTable t, void *img) {
+    const ReqDesc &r = t.r[blockIdx.y];
+    const int npairs = (r.nint + 1) >> 1;
+    const int64_t work = (int64_t)r.nwires * npairs;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < work;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int w = (int)(i / npairs);
+        const int bp = (int)(i - (int64_t)w * npairs);
+        const int b = 2 * bp;
+        const float *src = r.adc + (int64_t)w * r.ld + 6 * b;
+        const bool two = (b + 1) < r.nint;
+        const float4 x0 = __ldcs(reinterpret_cast<const float4 *>(src));
+        const float2 x1 = __ldcs(reinterpret_cast<const float2 *>(src + 4));
+        const float v0 = interval_sum(x0.x, x0.y, x0.z, x0.w, x1.x, x1.y);
+        float v1 = 0.0f;
+        if (two) {
+            const float2 x2 = __ldcs(reinterpret_cast<const float2 *>(src + 6));
+            const float4 x3 = __ldcs(reinterpret_cast<const float4 *>(src + 8));
+            v1 = interval_sum(x2.x, x2.y, x3.x, x3.y, x3.z, x3.w);
+        }
+        store2<FMT>(img, r.d_off + (int64_t)w * r.pitch + b, v0, v1, two);
+    }
+}
+
+template <int FMT>
+struct Elem;
+template <>
+struct Elem<EMTK_PATCH_F32> {
+    using T = float;
+};
+template <>
+struct Elem<EMTK_PATCH_BF16> {
+    using T = unsigned short;
+};
+template <>
+struct Elem<EMTK_PATCH_F16> {
+    using T = unsigned short;
+};
+
+__device__ __forceinline__ int find_request(const ReqTable &t, int64_t g) {
+    int lo = 0, hi = t.n - 1;
+    while (lo < hi) {  // last request with hit_begin <= g
+        const int mid = (lo + hi + 1) >> 1;
+        if (t.r[mid].hit_begin <= g)
+            lo = mid;
+        else
+            hi = mid - 1;
+    }
+    return lo;
+}
+
+__device__ __forceinline__ int64_t floor_div6(int64_t a) {
+    int64_t q = a / 6;
+    if ((a % 6) != 0 && a < 0) q -= 1;
+    return q;
+}
+
+// One block per hit: 48 rows x (48 / V) vectors of V elements (16 bytes).
+template <int FMT>
+__global__ void __launch_bounds__(288) gather_kernel(const __grid_constant__ ReqTable t, const void *img,
+                                                     int64_t g0, void *patches, float **dest,
+                                                     int out_stride) {
+    using T = typename Elem<FMT>::T;
+    constexpr int V = 16 / sizeof(T);
+    constexpr int CH = kPatch / V;
+    const int64_t local = blockIdx.x;
+    const int64_t g = g0 + local;
+    const int ri = find_request(t, g);
+    const ReqDesc &r = t.r[ri];
+    const int64_t hloc = g - r.hit_begin;
+    const emtk_hit hit = r.hits[hloc];
+    const int64_t wc = hit.wire;
+    const int64_t bc = floor_div6(hit.tick);
+    const T *src = static_cast<const T *>(img) + r.d_off;
+    T *out = static_cast<T *>(patches) + local * kPatchElems;
+    if (dest != nullptr && threadIdx.x == 0) dest[local] = r.scores + hloc * out_stride;
+    for (int task = threadIdx.x; task < kPatch * CH; task += blockDim.x) {
+        const int row = task / CH;
+        const int c0 = (task - row * CH) * V;
+        const int64_t w = wc - kHalf + row;
+        union {
+            T e[V];
+            uint4 u;
+        } v;
+        const bool wire_ok = (w >= 0 && w < r.nwires);
+#pragma unroll
+        for (int e = 0; e < V; ++e) {
+            const int64_t b = bc - kHalf + c0 + e;
+            v.e[e] = (wire_ok && b >= 0 && b < r.nint) ? src[w * r.pitch + b] : T(0);
+        }
+        *reinterpret_cast<uint4 *>(out + row * kPatch + c0) = v.u;
+    }
+}
+
+template <int FMT>
+__global__ void convert_kernel(const float *src, void *dst, int64_t n) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        const float v = src[i];
+        if (FMT == EMTK_PATCH_BF16)
+            static_cast<__nv_bfloat16 *>(dst)[i] = __float2bfloat16_rn(v);
+        else
+            static_cast<__half *>(dst)[i] = __float2half_rn(v);
+    }
+}
+
+__global__ void fill_dest_kernel(float *scores, int stride, float **dest, int32_t n) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i < n) dest[i] = scores + (int64_t)i * stride;
+}
+
+}  // namespace
+
+cudaError_t launch_interval_images(const ReqTable &t, void *dimg, emtk_patch_format fmt, cudaStream_t s) {
+    int64_t most = 0;
+    for (int i = 0; i < t.n; ++i) {
+        const int64_t w = (int64_t)t.r[i].nwires * ((t.r[i].nint + 1) / 2);
+        most = w > most ? w : most;
+    }
+    if (most == 0 || t.n == 0) return cudaSuccess;
+    int64_t bx = (most + 255) / 256;
+    if (bx > 4096) bx = 4096;
+    dim3 grid((unsigned)bx, (unsigned)t.n);
+    if (fmt == EMTK_PATCH_F32)
+        interval_image_kernel<EMTK_PATCH_F32><<<grid, 256, 0, s>>>(t, dimg);
+    else if (fmt == EMTK_PATCH_BF16)
+        interval_image_kernel<EMTK_PATCH_BF16><<<grid, 256, 0, s>>>(t, dimg);
+    else
+        interval_image_kernel<EMTK_PATCH_F16><<<grid, 256, 0, s>>>(t, dimg);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_gather(const ReqTable &t, const void *dimg, emtk_patch_format fmt, int64_t g0, int32_t count,
+                          void *patches, float **dest, int out_stride, cudaStream_t s) {
+    if (count <= 0) return cudaSuccess;
+    if (fmt == EMTK_PATCH_F32)
+        gather_kernel<EMTK_PATCH_F32><<<count, 288, 0, s>>>(t, dimg, g0, patches, dest, out_stride);
+    else if (fmt == EMTK_PATCH_BF16)
+        gather_kernel<EMTK_PATCH_BF16><<<count, 288, 0, s>>>(t, dimg, g0, patches, dest, out_stride);
+    else
+        gather_kernel<EMTK_PATCH_F16><<<count, 288, 0, s>>>(t, dimg, g0, patches, dest, out_stride);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_convert_patches(const float *src, void *dst, emtk_patch_format fmt, int64_t n, cudaStream_t s) {
+    if (n <= 0) return cudaSuccess;
+    int64_t blocks = (n + 255) / 256;
+    if (blocks > 8192) blocks = 8192;
+    if (fmt == EMTK_PATCH_BF16)
+        convert_kernel<EMTK_PATCH_BF16><<<(unsigned)blocks, 256, 0, s>>>(src, dst, n);
+    else
+        convert_kernel<EMTK_PATCH_F16><<<(unsigned)blocks, 256, 0, s>>>(src, dst, n);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_fill_dest(float *scores, int out_stride, float **dest, int32_t n, cudaStream_t s) {
+    if (n <= 0) return cudaSuccess;
+    fill_dest_kernel<<<(n + 255) / 256, 256, 0, s>>>(scores, out_stride, dest, n);
+    return cudaGetLastError();
+}
+
+}  // namespace emtk

@@ -1,0 +1,109 @@
+"""Host-side checks of the C ABI that need no GPU: the library loads, exports
+every entry point include/emtk.h declares, and rejects bad arguments before
+touching the device."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+from paper_2009_04509_gb300 import emtk, synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "emtk.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2009_04509_gb300 import build
+    build.build()
+    return emtk.load_library()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"EMTK_API\s+[\w\s\*]+?\b(emtk_\w+)\s*\(", text)))
+
+
+def test_header_declares_the_abi():
+    names = declared_functions()
+    assert set(names) == set(emtk.EXPORTED)
+    for n in ("emtk_create", "emtk_infer", "emtk_infer_batch", "emtk_extract_patches", "emtk_infer_patches"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_library_exports_nothing_else(lib):
+    import subprocess
+    out = subprocess.run(["nm", "-D", "--defined-only", emtk.LIB_PATH], capture_output=True, text=True)
+    if out.returncode != 0:
+        pytest.skip("nm not available")
+    syms = {l.split()[-1] for l in out.stdout.splitlines() if " T " in l}
+    assert {s for s in syms if s.startswith("emtk_")} == set(declared_functions())
+
+
+def test_status_strings(lib):
+    for code in range(7):
+        s = emtk.status_string(code)
+        assert s and s != "unknown status"
+    assert emtk.status_string(99) == "unknown status"
+
+
+def test_default_options(lib):
+    o = emtk.emtk_default_options()
+    assert o.precision == emtk.EMTK_BF16 and o.max_hits == 65536 and o.debug_logits == 0
+    assert o.wait_timeout_ns == 2_000_000_000 and o.debug_stall == 0 and o.profile == 0
+
+
+def test_struct_layouts_match_header(lib):
+    # emtk_request: ptr, 2 x int32, int64, ptr, int32 (+pad), ptr
+    assert ctypes.sizeof(emtk.emtk_request) == 48
+    assert emtk.emtk_request.d_scores.offset == 40
+    assert ctypes.sizeof(emtk.emtk_options) == 32
+    assert ctypes.sizeof(emtk.emtk_weights) == 80
+    assert ctypes.sizeof(emtk.emtk_stats) == 176
+
+
+def test_argument_errors_without_device(lib):
+    null = None
+    assert lib.emtk_infer(null, None, 1, 1, 4, None, 0, None, None) == emtk.EMTK_ERR_ARG
+    assert lib.emtk_infer_batch(null, None, 0, None) == emtk.EMTK_ERR_ARG
+    assert lib.emtk_extract_patches(null, None, 1, 1, 4, None, 0, None, 0, None) == emtk.EMTK_ERR_ARG
+    assert lib.emtk_infer_patches(null, None, 0, None, None) == emtk.EMTK_ERR_ARG
+    assert lib.emtk_check(null, None) == emtk.EMTK_ERR_ARG
+    assert lib.emtk_get_stats(null, None) == emtk.EMTK_ERR_ARG
+    assert lib.emtk_destroy(null) == emtk.EMTK_OK
+    out = ctypes.c_void_p()
+    assert lib.emtk_create(None, None, 0, ctypes.byref(out)) == emtk.EMTK_ERR_ARG and not out.value
+    w = synth.he_normal_weights(0, dims=dict(P=6, R=3, F=2, N1=2, N2=2, NC=3))
+    keep = {k: np.ascontiguousarray(v, np.float32) for k, v in w.items()}
+    ws = emtk.emtk_weights(**{k: v.ctypes.data_as(ctypes.POINTER(ctypes.c_float)) for k, v in keep.items()})
+    o = emtk.emtk_default_options()
+    o.precision = 7
+    assert lib.emtk_create(ctypes.byref(ws), ctypes.byref(o), 0, ctypes.byref(out)) == emtk.EMTK_ERR_ARG
+    o = emtk.emtk_default_options()
+    o.max_hits = 0
+    assert lib.emtk_create(ctypes.byref(ws), ctypes.byref(o), 0, ctypes.byref(out)) == emtk.EMTK_ERR_ARG
+    o = emtk.emtk_default_options()
+    o.precision = emtk.EMTK_TF32
+    assert lib.emtk_create(ctypes.byref(ws), ctypes.byref(o), 0, ctypes.byref(out)) == emtk.EMTK_ERR_UNSUPPORTED
+    assert lib.emtk_create(ctypes.byref(ws), None, -1, ctypes.byref(out)) == emtk.EMTK_ERR_ARG
+
+
+def test_create_without_gpu_reports_cuda_error(lib):
+    torch = pytest.importorskip("torch")
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    with pytest.raises(emtk.EmtkError) as e:
+        emtk.emtk_create(synth.he_normal_weights(0), precision="bf16")
+    assert e.value.status == emtk.EMTK_ERR_CUDA
+
+
+def test_missing_library_fails_loudly(tmp_path):
+    with pytest.raises(RuntimeError, match="no CPU fallback"):
+        emtk.load_library(str(tmp_path / "libemtk.so"))

@@ -1,0 +1,320 @@
+"""GPU parity: the CUDA path through the C ABI against the CPU oracle on the
+same seeded inputs.
+
+Bars (written here, derived in the design notes):
+* patch cut: bit-exact (fp32), and bit-exact after round-to-nearest-even for
+  the 16-bit formats;
+* fp32 network: max |score difference| <= 1e-3 against the fp64 oracle;
+* 16-bit network: >= 99.5% argmax agreement with the fp64 oracle, max |score
+  difference| <= 2e-2 against the oracle that rounds the same operands to the
+  same 16-bit format, and <= 2e-2 against the fp64 oracle on unsaturated
+  inputs (ADC / 100, biases N(0, 0.1)).  On raw ADC with He-normal weights
+  the network saturates (logits up to ~200) and the 16-bit operand rounding
+  alone moves scores of near-tie hits by more than 2e-2, in any
+  implementation, so there the fp64 bar is argmax agreement.
+"""
+import numpy as np
+import pytest
+
+import oracle
+from paper_2009_04509_gb300 import synth
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+TOL_FP32 = 1e-3
+TOL_16 = 2e-2
+ARGMAX_MIN = 0.995
+SAMPLE = 256
+
+
+@pytest.fixture(scope="module")
+def emtk():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2009_04509_gb300 import build, emtk as m
+    build.build()
+    oracle.build()
+    return m
+
+
+@pytest.fixture(scope="module")
+def weights():
+    return synth.he_normal_weights(0)
+
+
+@pytest.fixture(scope="module")
+def weights_b():
+    return synth.he_normal_weights(0, bias_std=0.1)
+
+
+_ctx_cache = {}
+
+
+@pytest.fixture(scope="module")
+def ctx_factory(emtk):
+    made = []
+
+    def make(w, precision, **kw):
+        key = (id(w), precision, tuple(sorted(kw.items())))
+        if key not in _ctx_cache:
+            _ctx_cache[key] = emtk.emtk_create(w, precision=precision, debug_logits=True, **kw)
+            made.append(key)
+        return _ctx_cache[key]
+
+    yield make
+    for k in made:
+        emtk.emtk_destroy(_ctx_cache.pop(k))
+
+
+def dev(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def run_infer(emtk, ctx, plane):
+    scores = torch.full((plane.nhits, 8), float("nan"), dtype=torch.float32, device="cuda")
+    emtk.emtk_infer(ctx, dev(plane.adc), plane.nticks, dev(plane.hits), scores)
+    assert emtk.emtk_check(ctx) == emtk.EMTK_OK
+    return scores.cpu().numpy().astype(np.float64)
+
+
+def adversarial_hits(nwires, nticks, rng):
+    edge = [[0, 0], [nwires - 1, nticks - 1], [0, nticks - 1], [nwires - 1, 0], [-100, 300], [20, 10_000_000],
+            [5, -7], [5, -6], [5, -1], [nwires + 23, 50], [nwires + 24, 50], [-24, 100], [-25, 100],
+            [nwires // 2, nticks], [nwires // 2, nticks + 143], [nwires // 2, nticks + 144]]
+    rand = np.stack([rng.integers(-60, nwires + 60, 40), rng.integers(-400, nticks + 400, 40)], 1)
+    h = np.concatenate([np.array(edge), rand]).astype(np.int32)
+    return np.concatenate([h, h[:4]])  # duplicates
+
+
+def check_16bit(got, emu, ref, tol=TOL_16):
+    d_emu = np.abs(got[:, :4] - emu).max()
+    agree = (got[:, :3].argmax(1) == ref[:, :3].argmax(1)).mean()
+    assert d_emu <= tol, f"max |score - emulated oracle| = {d_emu}"
+    assert agree >= ARGMAX_MIN, f"argmax agreement {agree}"
+    return d_emu, agree
+
+
+def check_invariants(got):
+    s = got[:, :4]
+    assert np.all(np.isfinite(s))
+    assert np.all(np.abs(s[:, :3].sum(1) - 1.0) <= 1e-5)
+    assert np.all((s >= 0.0) & (s <= 1.0))
+
+
+# ------------------------------------------------------------- patch cut
+@pytest.mark.parametrize("fmt", ["f32", "bf16", "fp16"])
+def test_extract_bit_exact(emtk, ctx_factory, weights, fmt):
+    rng = np.random.default_rng(1)
+    plane = synth.single_plane(seed=0)
+    hits = np.concatenate([plane.hits, adversarial_hits(plane.nwires, plane.nticks, rng)])
+    ctx = ctx_factory(weights, "bf16")
+    dt = torch.float32 if fmt == "f32" else torch.int16
+    out = torch.zeros((hits.shape[0], 48, 48), dtype=dt, device="cuda")
+    emtk.emtk_extract_patches(ctx, dev(plane.adc), plane.nticks, dev(hits), out, fmt)
+    assert emtk.emtk_check(ctx) == emtk.EMTK_OK
+    want = oracle.extract_patches(plane.adc, plane.nticks, hits)
+    got = out.cpu().numpy()
+    if fmt == "f32":
+        assert np.array_equal(got.view(np.uint32), want.view(np.uint32))
+    elif fmt == "bf16":
+        assert np.array_equal(got.view(np.uint16), oracle.round_bf16(want))
+    else:
+        assert np.array_equal(got.view(np.uint16), oracle.round_fp16(want).astype(np.float16).view(np.uint16))
+
+
+def test_extract_ragged_plane(emtk, ctx_factory, weights):
+    """nticks % 6 != 0, ld > nticks with poison beyond nticks, odd wire count."""
+    rng = np.random.default_rng(2)
+    nwires, nticks, ld = 37, 5997, 6004
+    adc = np.full((nwires, ld), 1e30, np.float32)
+    adc[:, :nticks] = (rng.standard_normal((nwires, nticks)) * 40).astype(np.float32)
+    hits = adversarial_hits(nwires, nticks, rng)
+    ctx = ctx_factory(weights, "bf16")
+    out = torch.zeros((hits.shape[0], 48, 48), dtype=torch.float32, device="cuda")
+    emtk.emtk_extract_patches(ctx, dev(adc), nticks, dev(hits), out, "f32")
+    assert emtk.emtk_check(ctx) == emtk.EMTK_OK
+    want = oracle.extract_patches(adc, nticks, hits)
+    assert np.array_equal(out.cpu().numpy().view(np.uint32), want.view(np.uint32))
+
+
+def test_extract_empty_and_errors(emtk, ctx_factory, weights):
+    ctx = ctx_factory(weights, "bf16")
+    plane = synth.single_plane(seed=0, nhits=4, nticks=600)
+    adc = dev(plane.adc)
+    empty = torch.zeros((0, 2), dtype=torch.int32, device="cuda")
+    out = torch.zeros((1, 48, 48), device="cuda")
+    emtk.emtk_extract_patches(ctx, adc, plane.nticks, empty, out, "f32")
+    lib = emtk.load_library()
+    hits = dev(plane.hits)
+    # misaligned plane pointer and bad leading dimension are refused up front
+    assert lib.emtk_extract_patches(ctx, adc.data_ptr() + 4, plane.nwires, plane.nticks, plane.ld, hits.data_ptr(),
+                                    4, out.data_ptr(), 0, None) == emtk.EMTK_ERR_ALIGN
+    assert lib.emtk_extract_patches(ctx, adc.data_ptr(), plane.nwires, plane.nticks, plane.nticks - 1,
+                                    hits.data_ptr(), 4, out.data_ptr(), 0, None) == emtk.EMTK_ERR_ARG
+    assert lib.emtk_extract_patches(ctx, adc.data_ptr(), plane.nwires, plane.nticks, plane.ld, hits.data_ptr(),
+                                    4, out.data_ptr(), 9, None) == emtk.EMTK_ERR_ARG
+    assert emtk.emtk_check(ctx) == emtk.EMTK_OK
+
+
+# ------------------------------------------------------------- network
+def test_fp32_single_plane(emtk, ctx_factory, weights):
+    plane = synth.single_plane(seed=0)
+    got = run_infer(emtk, ctx_factory(weights, "fp32"), plane)
+    lo, ref = oracle.forward(oracle.extract_patches(plane.adc, plane.nticks, plane.hits), weights)
+    assert np.abs(got[:, :4] - ref).max() <= TOL_FP32
+    assert np.abs(got[:, 4:] - lo).max() <= 1e-3 * max(1.0, np.abs(lo).max())
+    check_invariants(got)
+
+
+def test_fp32_unsaturated(emtk, ctx_factory, weights_b):
+    plane = synth.scaled(synth.single_plane(seed=3), 0.01)
+    got = run_infer(emtk, ctx_factory(weights_b, "fp32"), plane)
+    _, ref = oracle.forward(oracle.extract_patches(plane.adc, plane.nticks, plane.hits), weights_b)
+    assert np.abs(got[:, :4] - ref).max() <= TOL_FP32
+
+
+@pytest.mark.parametrize("prec", ["bf16", "fp16"])
+def test_16bit_single_plane(emtk, ctx_factory, weights, prec):
+    plane = synth.single_plane(seed=0)
+    got = run_infer(emtk, ctx_factory(weights, prec), plane)
+    p = oracle.extract_patches(plane.adc, plane.nticks, plane.hits)
+    _, ref = oracle.forward(p, weights)
+    _, emu = oracle.forward(p, weights, emulate=prec)
+    check_16bit(got, emu, ref)
+    check_invariants(got)
+
+
+@pytest.mark.parametrize("prec", ["bf16", "fp16"])
+def test_16bit_unsaturated_meets_fp64_bar(emtk, ctx_factory, weights_b, prec):
+    plane = synth.scaled(synth.single_plane(seed=4), 0.01)
+    got = run_infer(emtk, ctx_factory(weights_b, prec), plane)
+    _, ref = oracle.forward(oracle.extract_patches(plane.adc, plane.nticks, plane.hits), weights_b)
+    assert np.abs(got[:, :4] - ref).max() <= TOL_16
+    assert (got[:, :3].argmax(1) == ref[:, :3].argmax(1)).mean() >= ARGMAX_MIN
+
+
+@pytest.mark.parametrize("n", [1, 127, 128, 129, 383])
+def test_tile_edges(emtk, ctx_factory, weights, n):
+    """Hit counts that are not multiples of the 128-hit tile, including one."""
+    plane = synth.single_plane(seed=5, nhits=n, nticks=1200)
+    got = run_infer(emtk, ctx_factory(weights, "bf16"), plane)
+    p = oracle.extract_patches(plane.adc, plane.nticks, plane.hits)
+    _, ref = oracle.forward(p, weights)
+    _, emu = oracle.forward(p, weights, emulate="bf16")
+    assert np.abs(got[:, :4] - emu).max() <= TOL_16
+    check_invariants(got)
+
+
+def test_edge_hits_network(emtk, ctx_factory, weights):
+    """Hits on plane corners, outside it and duplicated run through the network."""
+    rng = np.random.default_rng(6)
+    base = synth.single_plane(seed=6, nhits=8, nticks=1200)
+    hits = adversarial_hits(base.nwires, base.nticks, rng)
+    plane = synth.Plane(adc=base.adc, nticks=base.nticks, hits=hits, kind=np.zeros(hits.shape[0], np.int8))
+    for prec in ("fp32", "bf16"):
+        got = run_infer(emtk, ctx_factory(weights, prec), plane)
+        p = oracle.extract_patches(plane.adc, plane.nticks, plane.hits)
+        _, ref = oracle.forward(p, weights)
+        if prec == "fp32":
+            assert np.abs(got[:, :4] - ref).max() <= TOL_FP32
+        else:
+            _, emu = oracle.forward(p, weights, emulate="bf16")
+            assert np.abs(got[:, :4] - emu).max() <= TOL_16
+        # identical hits give identical rows
+        n0 = hits.shape[0] - 4
+        assert np.array_equal(got[n0:], got[:4])
+
+
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+def test_infer_patches_lognormal(emtk, ctx_factory, weights, prec):
+    """Network only, on pre-cut fp32 patches (70% zeros, lognormal)."""
+    x = synth.inference_patches(300, seed=7)
+    scores = torch.zeros((300, 8), device="cuda")
+    ctx = ctx_factory(weights, prec)
+    emtk.emtk_infer_patches(ctx, dev(x), scores)
+    assert emtk.emtk_check(ctx) == emtk.EMTK_OK
+    got = scores.cpu().numpy().astype(np.float64)
+    _, ref = oracle.forward(x, weights)
+    if prec == "fp32":
+        assert np.abs(got[:, :4] - ref).max() <= TOL_FP32
+    else:
+        _, emu = oracle.forward(x, weights, emulate="bf16")
+        check_16bit(got, emu, ref)
+
+
+def test_batch_matches_single_calls(emtk, ctx_factory, weights):
+    planes = synth.apa(seed=8, hits=(300, 250, 0), n_tracks=5, n_showers=2)
+    ctx = ctx_factory(weights, "bf16")
+    items, outs = [], []
+    for p in planes:
+        s = torch.full((p.nhits, 8), float("nan"), device="cuda")
+        items.append((dev(p.adc), p.nticks, dev(p.hits), s))
+        outs.append(s)
+    emtk.emtk_infer_batch(ctx, items)
+    assert emtk.emtk_check(ctx) == emtk.EMTK_OK
+    for p, s in zip(planes, outs):
+        if p.nhits == 0:
+            continue
+        single = run_infer(emtk, ctx, p)
+        b = s.cpu().numpy().astype(np.float64)
+        assert np.abs(b[:, :4] - single[:, :4]).max() <= 1e-4
+        pp = oracle.extract_patches(p.adc, p.nticks, p.hits)
+        _, emu = oracle.forward(pp, weights, emulate="bf16")
+        assert np.abs(b[:, :4] - emu).max() <= TOL_16
+
+
+def test_deterministic(emtk, ctx_factory, weights):
+    plane = synth.single_plane(seed=9, nhits=500, nticks=1200)
+    ctx = ctx_factory(weights, "bf16")
+    a = run_infer(emtk, ctx, plane)
+    b = run_infer(emtk, ctx, plane)
+    assert np.array_equal(a, b)
+
+
+def test_chunked_call_matches(emtk, ctx_factory, weights):
+    """A context with a small workspace processes a large call in chunks."""
+    plane = synth.single_plane(seed=10, nhits=700, nticks=1200)
+    small = ctx_factory(weights, "bf16", max_hits=256)
+    got = run_infer(emtk, small, plane)
+    p = oracle.extract_patches(plane.adc, plane.nticks, plane.hits)
+    _, emu = oracle.forward(p, weights, emulate="bf16")
+    assert np.abs(got[:, :4] - emu).max() <= TOL_16
+    st = emtk.emtk_get_stats(small)
+    assert st["chunks"] >= 3
+
+
+def test_full_event_sampled(emtk, ctx_factory, weights):
+    """The full 18-plane event (60,000 hits) in one batched call, as the
+    benchmark runs it; a sample of hits is checked against the oracle and
+    every hit against the output invariants."""
+    planes = synth.full_event(seed=0)
+    ctx = ctx_factory(weights, "bf16")
+    items, outs = [], []
+    for p in planes:
+        s = torch.full((p.nhits, 8), float("nan"), device="cuda")
+        items.append((dev(p.adc), p.nticks, dev(p.hits), s))
+        outs.append(s)
+    emtk.emtk_infer_batch(ctx, items)
+    assert emtk.emtk_check(ctx) == emtk.EMTK_OK
+    got = [s.cpu().numpy().astype(np.float64) for s in outs]
+    check_invariants(np.concatenate(got))
+    rng = np.random.default_rng(11)
+    per = SAMPLE // len(planes) + 1
+    g_all, e_all, r_all = [], [], []
+    for p, g in zip(planes, got):
+        idx = rng.choice(p.nhits, per, replace=False)
+        pp = oracle.extract_patches(p.adc, p.nticks, p.hits[idx])
+        _, ref = oracle.forward(pp, weights)
+        _, emu = oracle.forward(pp, weights, emulate="bf16")
+        g_all.append(g[idx])
+        e_all.append(emu)
+        r_all.append(ref)
+    check_16bit(np.concatenate(g_all), np.concatenate(e_all), np.concatenate(r_all))
+    # patch cut at full plane size, sampled hits
+    p = planes[2]
+    idx = rng.choice(p.nhits, 64, replace=False)
+    out = torch.zeros((64, 48, 48), device="cuda")
+    emtk.emtk_extract_patches(ctx, dev(p.adc), p.nticks, dev(p.hits[idx]), out, "f32")
+    want = oracle.extract_patches(p.adc, p.nticks, p.hits[idx])
+    assert np.array_equal(out.cpu().numpy().view(np.uint32), want.view(np.uint32))
