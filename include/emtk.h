@@ -170,6 +170,32 @@ EMTK_API emtk_status emtk_extract_patches(emtk_ctx *ctx, const float *d_adc, int
                                  int64_t ld, const emtk_hit *d_hits, int32_t nhits, void *d_patches,
                                  emtk_patch_format fmt, emtk_stream stream);
 
+/* Size of the fixed device array behind emtk_extract_patches_static. */
+#define EMTK_STATIC_SCRATCH_BYTES (4u << 20)
+
+/* The patch cut of emtk_extract_patches for callers that cannot allocate
+ * device memory.  The paper has no counterpart; it is a service to callers
+ * whose device memory is already owned by another allocator (a framework's
+ * caching pool, a budget fixed at start-up) or that must avoid the
+ * device-wide synchronisation cudaMalloc / cudaFree can cause.  It takes no
+ * context (creating one allocates) and calls no allocating routine.
+ *   - Same arguments and output as emtk_extract_patches, on the current
+ *     device.
+ *   - Its scratch is one fixed array of EMTK_STATIC_SCRATCH_BYTES in the
+ *     library's static device memory, held by every GPU that loads the
+ *     library until the process exits.  The plane's interval image must fit:
+ *     nwires * ((nticks/6 rounded up to a multiple of 8)) * (4 for F32, 2 for
+ *     BF16/F16) <= EMTK_STATIC_SCRATCH_BYTES, else EMTK_ERR_ARG and nothing is
+ *     enqueued (a 960 x 6000 plane fits in every format).
+ *   - The first call on each device looks up the array's device address;
+ *     make that first call before any stream capture.
+ *   - All calls share the array.  Calls that overlap on the GPU (two streams,
+ *     two threads) race; serialise them.  Nothing needs clearing between
+ *     calls: every interval a call reads, that call wrote. */
+EMTK_API emtk_status emtk_extract_patches_static(const float *d_adc, int32_t nwires, int32_t nticks, int64_t ld,
+                                                 const emtk_hit *d_hits, int32_t nhits, void *d_patches,
+                                                 emtk_patch_format fmt, emtk_stream stream);
+
 /* Network only (Sec. 2.2) on pre-cut fp32 patches [n][48][48] -> d_scores. */
 EMTK_API emtk_status emtk_infer_patches(emtk_ctx *ctx, const float *d_patches, int32_t n, float *d_scores,
                                emtk_stream stream);

@@ -24,7 +24,8 @@ KERNELS = ("intervals", "gather", "network", "head", "convert")
 
 EXPORTED = ("emtk_default_options", "emtk_create", "emtk_destroy", "emtk_infer", "emtk_infer_batch",
             "emtk_extract_patches", "emtk_infer_patches", "emtk_check", "emtk_get_stats",
-            "emtk_status_string")
+            "emtk_status_string", "emtk_extract_patches_static")
+EMTK_STATIC_SCRATCH_BYTES = 4 << 20
 
 _vp = ctypes.c_void_p
 _fp = ctypes.POINTER(ctypes.c_float)
@@ -83,6 +84,9 @@ def load_library(path: str | None = None):
     lib.emtk_infer_patches.argtypes = [_vp, _vp, ctypes.c_int32, _vp, _vp]
     lib.emtk_check.argtypes = [_vp, _vp]
     lib.emtk_get_stats.argtypes = [_vp, ctypes.POINTER(emtk_stats)]
+    lib.emtk_extract_patches_static.argtypes = [_vp, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64, _vp,
+                                                ctypes.c_int32, _vp, ctypes.c_int, _vp]
+    lib.emtk_extract_patches_static.restype = ctypes.c_int
     lib.emtk_status_string.argtypes = [ctypes.c_int]
     lib.emtk_status_string.restype = ctypes.c_char_p
     for name in ("emtk_create", "emtk_destroy", "emtk_infer", "emtk_infer_batch", "emtk_extract_patches",
@@ -188,6 +192,16 @@ def emtk_extract_patches(ctx, adc, nticks: int, hits, patches, fmt: str = "f32",
     _check(load_library().emtk_extract_patches(ctx, _ptr(adc), int(nwires), int(nticks), int(ld), _ptr(hits),
                                                int(hits.shape[0]), _ptr(patches), PATCH_FORMATS[fmt],
                                                _stream(stream)), "emtk_extract_patches")
+
+
+def emtk_extract_patches_static(adc, nticks: int, hits, patches, fmt: str = "f32", stream=None) -> None:
+    """The patch cut without a context and without any device allocation, for
+    callers that cannot allocate; its scratch is a fixed 4 MiB array in the
+    library (see include/emtk.h for the size limit and the sharing rules)."""
+    nwires, ld = adc.shape
+    _check(load_library().emtk_extract_patches_static(_ptr(adc), int(nwires), int(nticks), int(ld), _ptr(hits),
+                                                      int(hits.shape[0]), _ptr(patches), PATCH_FORMATS[fmt],
+                                                      _stream(stream)), "emtk_extract_patches_static")
 
 
 def emtk_infer_patches(ctx, patches, scores, stream=None) -> None:
