@@ -3,22 +3,27 @@
 // the 92,928 conv activations of a hit never leave the SM.
 //
 // One CTA = 128 hits (one TMEM lane each) x one segment of the dense-1 input
-// dimension, walked conv position by conv position (p = y*44 + x; the
-// dense-1 input index is p*48 + c, the paper's channels-last flatten).
-// Per position:
-//   builder warps   write the hit's 5x5 im2col row (25 taps, two bias taps
-//                   of 1.0, zero padding to K = 32) into TMEM;
-//   MMA thread      conv MMA  D[128 x 48] = A_tmem[128 x 32] * Bconv[32 x 48]
-//                   (the conv bias rides on the two constant taps);
-//   epilogue warps  ReLU + round the conv tile to 16 bit, written back into
-//                   TMEM over the conv accumulator;
-//   MMA thread      dense-1 MMA  ACC[128 x 128] += A_tmem[128 x 48] * W1[48 x 128]
-//                   with W1 streamed through a 4-deep TMA ring in shared
-//                   memory (128-byte swizzle, 4 positions per stage).
-// Both MMAs take their A operand from tensor memory; shared memory only
-// carries the W1 stream and the conv weights.  Every wait is bounded: on
-// timeout the CTA raises an abort flag, sets bit 0 of the status word, waits
-// for its in-flight copies and MMAs, frees TMEM and returns.
+// dimension.  Conv positions p = y*44 + x are walked in quads (4 positions
+// of one row; the dense-1 input index is p*48 + c, the paper's channels-last
+// flatten), and each quad is two position pairs (x, x+1):
+//   builder warps   write, per hit, the 5 x 6 window of a pair (30 taps) and
+//                   two bias taps of 1.0 as one 32-wide im2col row into a
+//                   swizzled shared-memory tile (one 128-byte row per hit and
+//                   quad);
+//   MMA warp        conv MMA  D[128 x 96] = A_smem[128 x 32] * Bpair[32 x 96]:
+//                   columns 0-47 are the 48 filters at x (tap column 5 has a
+//                   zero weight), columns 48-95 the filters at x+1 (tap
+//                   column 0 zero); the conv bias rides on the bias taps;
+//   epilogue warps  ReLU + round the 128 x 96 conv tile to 16 bit, written
+//                   back into TMEM over it;
+//   MMA warp        dense-1  ACC[128 x 128] += A_tmem[128 x 96] * W1[96 x 128],
+//                   W1 streamed by TMA through a 3-stage ring (one quad, 48 KB,
+//                   per stage, 128-byte swizzle).
+// The MMA stream alternates [conv of quad q (2 pairs)] [dense-1 of quad q-1
+// (12 MMAs into one accumulator)], which keeps the tensor pipe busy while a
+// conv tile makes its round trip through the epilogue.  Every wait is
+// bounded: on timeout the CTA raises an abort flag, sets bit 0 of the status
+// word, waits for its in-flight copies and MMAs, frees TMEM and returns.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
@@ -32,35 +37,38 @@ namespace emtk {
 namespace {
 
 constexpr int kThreadsTC = 320;  // warp 0 TMA, warp 1 MMA, warps 2-5 builder, warps 6-9 epilogue
-constexpr int kStages = 6;       // TMEM stages, one conv position each
-constexpr int kW1Stages = 4;     // shared-memory stages of W1
-constexpr int kPosPerW1 = 4;     // conv positions per W1 stage
-constexpr int kW1Steps = kPos / kPosPerW1;                  // 484
+constexpr int kW1Stages = 3;     // shared-memory stages of W1 (one quad each)
+constexpr int kImBufs = 3;       // shared-memory im2col tiles (one quad each)
+constexpr int kSlots = 4;        // TMEM conv/activation slots (one pair each)
+constexpr int kPosPerW1 = 4;     // conv positions per W1 stage = per quad
+constexpr int kW1Steps = kPos / kPosPerW1;                  // 484 quads
 constexpr int kW1Box = 64;                                   // K elements per TMA box (128 B)
 constexpr int kW1BoxBytes = kW1Box * kN1 * 2;                // 16384
 constexpr int kBoxesPerStage = kPosPerW1 * kF / kW1Box;      // 3
 constexpr int kW1StageBytes = kBoxesPerStage * kW1BoxBytes;  // 49152
 constexpr int kKBlocks = kFc1In / kW1Box;                    // 1452
-constexpr int kConvK = 32;                                   // 25 taps + 2 bias taps + 5 zeros
-constexpr int kConvBBytes = kF * 128;                        // 48 rows of one 128-byte swizzle span
+constexpr int kPairN = 2 * kF;                               // 96 conv outputs per pair
+constexpr int kConvK = 32;                                   // 30 window taps + 2 bias taps
+constexpr int kImBytes = 128 * 128;                          // 128 hits x (2 pairs x 32 taps x 2 B)
+constexpr int kConvBBytes = kPairN * 128;                    // 96 rows of one 128-byte swizzle span
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kAccCol = 0;
-constexpr uint32_t kStageCol0 = 128;
-constexpr uint32_t kStageCols = 64;
-constexpr uint32_t kIm2colOff = 48;
-constexpr int kLag = 2;          // dense-1 of position p is issued after the conv of p + 2
+constexpr uint32_t kAccCol = 0;                              // dense-1 accumulator, 128 fp32 columns
+constexpr uint32_t kSlotCol0 = 128;                          // conv fp32 tile of a pair, then its activations
+constexpr uint32_t kSlotCols = kPairN;
 
 constexpr int kOffW1 = 0;
-constexpr int kOffConvB = kOffW1 + kW1Stages * kW1StageBytes;
+constexpr int kOffIm = kOffW1 + kW1Stages * kW1StageBytes;
+constexpr int kOffConvB = kOffIm + kImBufs * kImBytes;
 constexpr int kOffBar = kOffConvB + kConvBBytes;
 // barrier indices
 constexpr int kBarW1Full = 0;
 constexpr int kBarW1Empty = kBarW1Full + kW1Stages;
-constexpr int kBarIm2col = kBarW1Empty + kW1Stages;
-constexpr int kBarConv = kBarIm2col + kStages;
-constexpr int kBarAct = kBarConv + kStages;
-constexpr int kBarFree = kBarAct + kStages;
-constexpr int kBarAcc = kBarFree + kStages;
+constexpr int kBarImFull = kBarW1Empty + kW1Stages;  // im2col tile written (4 builder warps)
+constexpr int kBarImFree = kBarImFull + kImBufs;     // im2col tile read by its convs (MMA commit)
+constexpr int kBarConv = kBarImFree + kImBufs;       // conv tile of a pair done (MMA commit)
+constexpr int kBarAct = kBarConv + kSlots;           // activations written (4 epilogue warps)
+constexpr int kBarFree = kBarAct + kSlots;           // dense-1 of the slot's pair done (MMA commit)
+constexpr int kBarAcc = kBarFree + kSlots;
 constexpr int kBarStall = kBarAcc + 1;
 constexpr int kBarDrain = kBarStall + 1;
 constexpr int kNumBars = kBarDrain + 1;
@@ -69,7 +77,8 @@ constexpr int kOffAbort = kOffTmemSlot + 4;
 constexpr int kSmemUsed = kOffAbort + 4;
 constexpr int kSmemBytesTC = kSmemUsed + 1024;  // slack for 1024-byte alignment
 static_assert(kSmemBytesTC <= 232448, "shared memory budget");
-static_assert(kStageCol0 + kStages * kStageCols <= kTmemCols, "TMEM budget");
+static_assert(kSlotCol0 + kSlots * kSlotCols <= kTmemCols, "TMEM budget");
+static_assert(kQ % kPosPerW1 == 0, "quads do not straddle rows");
 
 // ------------------------------------------------------------ PTX helpers
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
@@ -110,8 +119,7 @@ struct Guard {
 // Waits for the phase of `parity` to complete.  Gives up (false) when the
 // CTA's abort flag is raised or after timeout_ns, raising the flag and the
 // status bit itself in the second case.
-__device__ __noinline__ bool wait_bounded(uint32_t bar, uint32_t parity, Guard g) {
-    if (mbar_try_wait(bar, parity)) return true;
+__device__ __noinline__ bool wait_slow(uint32_t bar, uint32_t parity, Guard g) {
     const uint64_t t0 = global_timer_ns();
     for (uint32_t i = 1;; ++i) {
         if (mbar_try_wait(bar, parity)) return true;
@@ -124,6 +132,11 @@ __device__ __noinline__ bool wait_bounded(uint32_t bar, uint32_t parity, Guard g
             }
         }
     }
+}
+
+__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, const Guard &g) {
+    if (mbar_try_wait(bar, parity)) return true;
+    return wait_slow(bar, parity, g);
 }
 
 // Lane 0 waits; the outcome is broadcast so the whole warp takes the same path.
@@ -154,6 +167,15 @@ __device__ __forceinline__ void mma_ts(uint32_t d, uint32_t a, uint64_t bdesc, u
         "setp.ne.b32 p, %4, 0;\n\t"
         "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d),
         "r"(a), "l"(bdesc), "r"(idesc), "r"(accum)
+        : "memory");
+}
+// D[tmem] (+)= A[smem desc] * B[smem desc], kind::f16, one CTA.
+__device__ __forceinline__ void mma_ss(uint32_t d, uint64_t adesc, uint64_t bdesc, uint32_t idesc, uint32_t accum) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accum)
         : "memory");
 }
 __device__ __forceinline__ void mma_commit(uint32_t bar) {
@@ -234,6 +256,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     const uint32_t base = (raw_u32 + 1023u) & ~1023u;
     uint8_t *gbase = smem_raw + (base - raw_u32);
     const uint32_t sW1 = base + kOffW1;
+    const uint32_t sIm = base + kOffIm;
     const uint32_t sConvB = base + kOffConvB;
     auto bar = [&](int i) -> uint32_t { return base + kOffBar + 8u * (uint32_t)i; };
     volatile uint32_t *tmem_slot = reinterpret_cast<volatile uint32_t *>(gbase + kOffTmemSlot);
@@ -243,16 +266,13 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     const int lane = threadIdx.x & 31;
     const int m_tile = blockIdx.x;
     const int seg = blockIdx.y;
-    const int j0 = (int)((int64_t)seg * kW1Steps / splits);
+    const int j0 = (int)((int64_t)seg * kW1Steps / splits);   // first quad
     const int j1 = (int)((int64_t)(seg + 1) * kW1Steps / splits);
-    const int nW1 = j1 - j0;
-    const int p0 = j0 * kPosPerW1;
-    const int p1 = j1 * kPosPerW1;
-    const int npos = p1 - p0;
+    const int nq = j1 - j0;                                     // quads in this segment
     const Guard guard{abort_flag, status, (int64_t)timeout_ns};
 
-    // ---- set-up: conv B operand into swizzled smem, barriers, TMEM
-    for (int idx = threadIdx.x; idx < kF * 8; idx += kThreadsTC) {
+    // ---- set-up: pair conv B operand into swizzled smem, barriers, TMEM
+    for (int idx = threadIdx.x; idx < kPairN * 8; idx += kThreadsTC) {
         const int row = idx >> 3, chunk = idx & 7;
         uint4 v = make_uint4(0u, 0u, 0u, 0u);
         if (chunk < kConvK / 8) v = __ldg(reinterpret_cast<const uint4 *>(convB_g + row * kConvK) + chunk);
@@ -263,8 +283,11 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
             mbar_init(bar(kBarW1Full + i), 1);
             mbar_init(bar(kBarW1Empty + i), 1);
         }
-        for (int i = 0; i < kStages; ++i) {
-            mbar_init(bar(kBarIm2col + i), 4);
+        for (int i = 0; i < kImBufs; ++i) {
+            mbar_init(bar(kBarImFull + i), 4);
+            mbar_init(bar(kBarImFree + i), 1);
+        }
+        for (int i = 0; i < kSlots; ++i) {
             mbar_init(bar(kBarConv + i), 1);
             mbar_init(bar(kBarAct + i), 4);
             mbar_init(bar(kBarFree + i), 1);
@@ -292,7 +315,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         if (lane == 0) {
             int issued = 0;
             bool ok = true;
-            for (int jj = 0; jj < nW1; ++jj) {
+            for (int jj = 0; jj < nq; ++jj) {
                 const int wj = jj % kW1Stages;
                 const uint32_t use = (uint32_t)(jj / kW1Stages);
                 if (jj >= kW1Stages && !wait_bounded(bar(kBarW1Empty + wj), (use - 1u) & 1u, guard)) {
@@ -322,54 +345,79 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         }
     } else if (warp == 1) {
         // ======================================================= MMA issuer
-        if (lane == 0) {
-            constexpr uint32_t idesc_conv = make_idesc(128, kF, FP16);
-            constexpr uint32_t idesc_fc1 = make_idesc(128, kN1, FP16);
-            const uint64_t convb_desc = sw128_desc(sConvB);
-            bool ok = true;
-            if (debug_stall) ok = wait_bounded(bar(kBarStall), 0u, guard);  // nothing arrives here
-            for (int k = 0; ok && k < npos + kLag; ++k) {
-                if (k < npos) {
-                    const int s = k % kStages;
-                    const uint32_t use = (uint32_t)(k / kStages);
-                    if (!wait_bounded(bar(kBarIm2col + s), use & 1u, guard)) {
+        // The whole warp walks the schedule; lane 0 issues every MMA and every
+        // commit, so each commit covers all earlier MMAs.  Iteration q: the
+        // convs of quad q (pairs 2q, 2q+1), then dense-1 of quad q-1.
+        constexpr uint32_t idesc_conv = make_idesc(128, kPairN, FP16);
+        constexpr uint32_t idesc_fc1 = make_idesc(128, kN1, FP16);
+        const uint64_t convb_desc = sw128_desc(sConvB);
+        bool ok = true;
+        if (debug_stall) ok = warp_wait(bar(kBarStall), 0u, guard, lane);  // nothing arrives here
+        for (int q = 0; ok && q <= nq; ++q) {
+            if (q < nq) {
+                const int ib = q % kImBufs;
+                if (!warp_wait(bar(kBarImFull + ib), (uint32_t)(q / kImBufs) & 1u, guard, lane)) {
+                    ok = false;
+                    break;
+                }
+                for (int pr = 0; pr < 2; ++pr) {
+                    const int pi = 2 * q + pr;
+                    const int s = pi % kSlots;
+                    // the slot's previous pair (pi - kSlots) has been read by its dense-1
+                    if (pi >= kSlots &&
+                        !warp_wait(bar(kBarFree + s), (uint32_t)(pi / kSlots - 1) & 1u, guard, lane)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t d = tmem + kStageCol0 + (uint32_t)s * kStageCols;
-                    mma_ts(d, d + kIm2colOff, convb_desc, idesc_conv, 0u);
-                    mma_ts(d, d + kIm2colOff + 8u, convb_desc + (32u >> 4), idesc_conv, 1u);
-                    mma_commit(bar(kBarConv + s));
+                    if (lane == 0) {
+                        const uint32_t d = tmem + kSlotCol0 + (uint32_t)s * kSlotCols;
+                        const uint64_t ad = sw128_desc(sIm + ib * kImBytes) + (uint64_t)((pr * 64) >> 4);
+                        mma_ss(d, ad, convb_desc, idesc_conv, 0u);
+                        mma_ss(d, ad + (32u >> 4), convb_desc + (32u >> 4), idesc_conv, 1u);
+                        mma_commit(bar(kBarConv + s));
+                    }
+                    __syncwarp();
                 }
-                const int qq = k - kLag;
-                if (qq >= 0) {
-                    const int sq = qq % kStages;
-                    const uint32_t uq = (uint32_t)(qq / kStages);
-                    const int jj = qq / kPosPerW1;
-                    const int wj = jj % kW1Stages;
-                    const int pin = qq % kPosPerW1;
-                    if (pin == 0 && !wait_bounded(bar(kBarW1Full + wj), (uint32_t)(jj / kW1Stages) & 1u, guard)) {
-                        ok = false;
-                        break;
-                    }
-                    if (!wait_bounded(bar(kBarAct + sq), uq & 1u, guard)) {
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
-                    const uint64_t wdesc = sw128_desc(sW1 + wj * kW1StageBytes);
-                    const uint32_t a = tmem + kStageCol0 + (uint32_t)sq * kStageCols;
-#pragma unroll
-                    for (int t = 0; t < 3; ++t) {
-                        const int step = pin * 3 + t;
-                        const uint64_t bd = wdesc + (uint64_t)(((step >> 2) * kW1BoxBytes + (step & 3) * 32) >> 4);
-                        mma_ts(tmem + kAccCol, a + 8u * t, bd, idesc_fc1, (qq > 0 || t > 0) ? 1u : 0u);
-                    }
-                    mma_commit(bar(kBarFree + sq));
-                    if (pin == kPosPerW1 - 1) mma_commit(bar(kBarW1Empty + wj));
-                }
+                if (!ok) break;
+                if (lane == 0) mma_commit(bar(kBarImFree + ib));
+                __syncwarp();
             }
+            const int qq = q - 1;
+            if (qq >= 0) {
+                const int wj = qq % kW1Stages;
+                if (!warp_wait(bar(kBarW1Full + wj), (uint32_t)(qq / kW1Stages) & 1u, guard, lane)) {
+                    ok = false;
+                    break;
+                }
+                const uint64_t wdesc = sw128_desc(sW1 + wj * kW1StageBytes);
+                for (int pr = 0; pr < 2; ++pr) {
+                    const int pi = 2 * qq + pr;
+                    const int s = pi % kSlots;
+                    if (!warp_wait(bar(kBarAct + s), (uint32_t)(pi / kSlots) & 1u, guard, lane)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    if (lane == 0) {
+                        const uint32_t a = tmem + kSlotCol0 + (uint32_t)s * kSlotCols;
+#pragma unroll
+                        for (int t = 0; t < 6; ++t) {
+                            const int step = pr * 6 + t;  // 16-wide K step inside the quad's 192
+                            const uint64_t bd =
+                                wdesc + (uint64_t)(((step >> 2) * kW1BoxBytes + (step & 3) * 32) >> 4);
+                            mma_ts(tmem + kAccCol, a + 8u * t, bd, idesc_fc1, (qq > 0 || step > 0) ? 1u : 0u);
+                        }
+                        mma_commit(bar(kBarFree + s));
+                    }
+                    __syncwarp();
+                }
+                if (!ok) break;
+                if (lane == 0) mma_commit(bar(kBarW1Empty + wj));
+                __syncwarp();
+            }
+        }
+        if (lane == 0) {
             if (ok) mma_commit(bar(kBarAcc));
             // every MMA issued so far completes before TMEM is released
             mma_commit(bar(kBarDrain));
@@ -377,20 +425,29 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
             while (!mbar_try_wait(bar(kBarDrain), 0u) && (int64_t)(global_timer_ns() - t0) < (int64_t)timeout_ns) {
             }
         }
+        __syncwarp();
     } else if (warp < 6) {
         // ================================================ im2col builder
-        const int q = warp & 3;
-        const int row = 32 * q + lane;
+        // Row r of an im2col tile (hit r) is 128 bytes: pair (x, x+1) in
+        // chunks 0-3, pair (x+2, x+3) in chunks 4-7; 16-byte chunk c sits at
+        // chunk c ^ (r & 7) (128-byte swizzle).  Tap t = 6i + j of a pair at x
+        // is patch pixel (y + i, x + j); taps 30 and 31 are 1.0.  Because x is
+        // even, taps (2k, 2k+1) are one aligned pixel pair of the patch row.
+        const int q4 = warp & 3;
+        const int row = 32 * q4 + lane;
         const int64_t hit = (int64_t)m_tile * 128 + row;
         const bool valid = hit < n;
         const uint4 *prow = reinterpret_cast<const uint4 *>(patches) + (valid ? hit : 0) * (kPatchElems / 8);
         const uint32_t one = FP16 ? 0x3C00u : 0x3F80u;
-        const uint32_t lane_tmem = tmem + ((uint32_t)(32 * q) << 16);
+        const uint32_t ones = one | (one << 16);
+        uint8_t *my_row = gbase + kOffIm + row * 128;
+        const int p0 = j0 * kPosPerW1;
+        const int p1 = j1 * kPosPerW1;
         const int y_first = p0 / kQ;
-        const int y_last = (p1 - 1) / kQ;
-        bool ok = npos > 0;
+        const int y_last = nq > 0 ? (p1 - 1) / kQ : y_first - 1;
+        bool ok = true;
         for (int y = y_first; ok && y <= y_last; ++y) {
-            uint32_t R[kK][24];
+            uint32_t R[kK][24];  // patch rows y..y+4 of this hit, 2 pixels per word
 #pragma unroll
             for (int i = 0; i < kK; ++i) {
 #pragma unroll
@@ -403,73 +460,73 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 }
             }
 #pragma unroll
-            for (int x = 0; x < kQ; ++x) {
-                const int p = y * kQ + x;
-                if (p < p0 || p >= p1) continue;
-                const int k = p - p0;
-                const int s = k % kStages;
-                const uint32_t use = (uint32_t)(k / kStages);
-                if (k >= kStages && !warp_wait(bar(kBarFree + s), (use - 1u) & 1u, guard, lane)) {
+            for (int xq = 0; xq < kQ / kPosPerW1; ++xq) {
+                const int quad = (y * kQ) / kPosPerW1 + xq;
+                if (quad < j0 || quad >= j1) continue;
+                const int k = quad - j0;
+                const int ib = k % kImBufs;
+                if (k >= kImBufs &&
+                    !warp_wait(bar(kBarImFree + ib), (uint32_t)(k / kImBufs - 1) & 1u, guard, lane)) {
                     ok = false;
                     break;
                 }
-                uint32_t v[16];
+                uint8_t *dst = my_row + ib * kImBytes;
 #pragma unroll
-                for (int pr = 0; pr < 13; ++pr) {
-                    const int t0 = 2 * pr, t1 = 2 * pr + 1;
-                    const int e0 = x + t0 % kK;
-                    const uint32_t sel_lo = (e0 & 1) ? 0x32u : 0x10u;
-                    const uint32_t lo = R[t0 / kK][e0 >> 1];
-                    if (t1 < kK * kK) {
-                        const int e1 = x + t1 % kK;
-                        const uint32_t sel = sel_lo | (((e1 & 1) ? 0x76u : 0x54u) << 8);
-                        v[pr] = __byte_perm(lo, R[t1 / kK][e1 >> 1], sel);
-                    } else {
-                        v[pr] = __byte_perm(lo, one, sel_lo | (0x54u << 8));  // tap 25 = 1.0
+                for (int c = 0; c < 8; ++c) {  // chunk c: pair c/4, taps 8(c%4) .. 8(c%4)+7
+                    const int x = 4 * xq + 2 * (c >> 2);
+                    uint32_t w[4];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const int kw = 4 * (c & 3) + e;  // word kw: taps 2kw, 2kw+1
+                        if (kw == 15) {
+                            w[e] = ones;
+                        } else {
+                            const int i = kw / 3, jp = kw % 3;  // row i, columns x + 2jp, x + 2jp + 1
+                            w[e] = R[i][(x >> 1) + jp];
+                        }
                     }
+                    *reinterpret_cast<uint4 *>(dst + ((c ^ (row & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
                 }
-                v[13] = one;  // tap 26 = 1.0, tap 27 = 0
-                v[14] = 0u;
-                v[15] = 0u;
-                tmem_st16<0>(lane_tmem + kStageCol0 + (uint32_t)s * kStageCols + kIm2colOff, v);
-                tmem_st_wait();
-                tc_fence_before();
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                 __syncwarp();
-                if (lane == 0) mbar_arrive(bar(kBarIm2col + s));
+                if (lane == 0) mbar_arrive(bar(kBarImFull + ib));
             }
         }
     } else {
         // ================================== conv epilogue + dense-1 store
-        const int q = warp & 3;
-        const int row = 32 * q + lane;
+        const int q4 = warp & 3;
+        const int row = 32 * q4 + lane;
         const int64_t hit = (int64_t)m_tile * 128 + row;
-        const uint32_t lane_tmem = tmem + ((uint32_t)(32 * q) << 16);
+        const uint32_t lane_tmem = tmem + ((uint32_t)(32 * q4) << 16);
         bool ok = true;
-        for (int k = 0; k < npos; ++k) {
-            const int s = k % kStages;
-            if (!warp_wait(bar(kBarConv + s), (uint32_t)(k / kStages) & 1u, guard, lane)) {
+        for (int pi = 0; pi < 2 * nq; ++pi) {
+            const int s = pi % kSlots;
+            if (!warp_wait(bar(kBarConv + s), (uint32_t)(pi / kSlots) & 1u, guard, lane)) {
                 ok = false;
                 break;
             }
             tc_fence_after();
-            const uint32_t d = lane_tmem + kStageCol0 + (uint32_t)s * kStageCols;
-            uint32_t f[48];
-            tmem_ld16<0>(d, f);
-            tmem_ld16<16>(d + 16u, f);
-            tmem_ld16<32>(d + 32u, f);
-            tmem_ld_wait();
-            reg_fence(f);
-            uint32_t o[24];
+            const uint32_t d = lane_tmem + kSlotCol0 + (uint32_t)s * kSlotCols;
 #pragma unroll
-            for (int i = 0; i < 24; ++i) o[i] = relu_pack<FP16>(f[2 * i], f[2 * i + 1]);
-            tmem_st16<0>(d, o);
-            tmem_st8<16>(d + 16u, o);
+            for (int h = 0; h < 2; ++h) {  // position x, then x+1: 48 fp32 -> 24 packed words
+                uint32_t f[48];
+                tmem_ld16<0>(d + 48u * h, f);
+                tmem_ld16<16>(d + 48u * h + 16u, f);
+                tmem_ld16<32>(d + 48u * h + 32u, f);
+                tmem_ld_wait();
+                reg_fence(f);
+                uint32_t o[24];
+#pragma unroll
+                for (int i = 0; i < 24; ++i) o[i] = relu_pack<FP16>(f[2 * i], f[2 * i + 1]);
+                tmem_st16<0>(d + 24u * h, o);
+                tmem_st8<16>(d + 24u * h + 16u, o);
+            }
             tmem_st_wait();
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(bar(kBarAct + s));
         }
-        if (ok && npos > 0 && warp_wait(bar(kBarAcc), 0u, guard, lane)) {
+        if (ok && nq > 0 && warp_wait(bar(kBarAcc), 0u, guard, lane)) {
             tc_fence_after();
             float *dst = partials + ((int64_t)seg * n_pad + hit) * kN1;
 #pragma unroll
@@ -535,13 +592,23 @@ cudaError_t prepare_tc_weights(DeviceWeights &w, const emtk_weights &hw, bool fp
         for (int nn = 0; nn < kN1; ++nn)
             for (int kk = 0; kk < kW1Box; ++kk)
                 tiles[((size_t)kb * kN1 + nn) * kW1Box + kk] = to16(hw.fc1_w[(size_t)(kb * kW1Box + kk) * kN1 + nn], fp16);
-    // conv B operand [48 filters][32]: taps 0..24, bias hi, bias lo, zeros
-    std::vector<uint16_t> cb((size_t)kF * kConvK, 0);
+    // pair conv B operand [96][32]: row f (< 48) is filter f at x, row 48 + f
+    // filter f at x + 1; tap t = 6i + j reads window column j; taps 30 and 31
+    // carry the bias split into a 16-bit head and a 16-bit remainder.
+    std::vector<uint16_t> cb((size_t)kPairN * kConvK, 0);
     for (int f = 0; f < kF; ++f) {
-        for (int t = 0; t < kK * kK; ++t) cb[f * kConvK + t] = to16(hw.conv_w[t * kF + f], fp16);
+        for (int i = 0; i < kK; ++i)
+            for (int j = 0; j < kK; ++j) {
+                const uint16_t wv = to16(hw.conv_w[(i * kK + j) * kF + f], fp16);
+                cb[(size_t)f * kConvK + 6 * i + j] = wv;              // position x: window columns 0..4
+                cb[(size_t)(kF + f) * kConvK + 6 * i + j + 1] = wv;   // position x+1: window columns 1..5
+            }
         const uint16_t hi = to16(hw.conv_b[f], fp16);
-        cb[f * kConvK + 25] = hi;
-        cb[f * kConvK + 26] = to16(hw.conv_b[f] - from16(hi, fp16), fp16);
+        const uint16_t lo = to16(hw.conv_b[f] - from16(hi, fp16), fp16);
+        for (int h = 0; h < 2; ++h) {
+            cb[(size_t)(h * kF + f) * kConvK + 30] = hi;
+            cb[(size_t)(h * kF + f) * kConvK + 31] = lo;
+        }
     }
     cudaError_t e = cudaMalloc(&w.w1_tiles, tiles.size() * 2);
     if (e != cudaSuccess) return e;
@@ -573,10 +640,9 @@ cudaError_t prepare_tc_weights(DeviceWeights &w, const emtk_weights &hw, bool fp
     return cudaSuccess;
 }
 
-// Splits of the dense-1 input (in W1 stages of 4 positions) so that
-// m_tiles x splits CTAs fill the SMs in few, even waves.  Time model per
-// wave: the segment's stages plus a fixed cost of about 6 stages (pipeline
-// fill and drain, partial-sum store).
+// Splits of the dense-1 input (in quads) so that m_tiles x splits CTAs fill
+// the SMs in few, even waves.  Time model per wave: the segment's quads plus
+// a fixed cost of about 6 quads (pipeline fill and drain, partial-sum store).
 int choose_splits_tc(int n, int sm_count, int max_splits) {
     const int m_tiles = (n + 127) / 128;
     int best = 1;
