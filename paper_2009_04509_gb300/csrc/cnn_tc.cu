@@ -36,7 +36,8 @@
 namespace emtk {
 namespace {
 
-constexpr int kThreadsTC = 320;  // warp 0 TMA, warp 1 MMA, warps 2-5 builder, warps 6-9 epilogue
+constexpr int kThreadsTC = 352;  // warp 0 TMA, warp 1 conv MMA, 2-5 builder, 6-9 epilogue, 10 dense-1 MMA
+constexpr int kFc1Warp = 10;
 constexpr int kW1Stages = 3;     // shared-memory stages of W1 (one quad each)
 constexpr int kImBufs = 3;       // shared-memory im2col tiles (one quad each)
 constexpr int kSlots = 4;        // TMEM conv/activation slots (one pair each)
@@ -294,7 +295,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         }
         mbar_init(bar(kBarAcc), 1);
         mbar_init(bar(kBarStall), 1);
-        mbar_init(bar(kBarDrain), 1);
+        mbar_init(bar(kBarDrain), 2);
         *abort_flag = 0u;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -343,83 +344,80 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 }
             }
         }
-    } else if (warp == 1) {
-        // ======================================================= MMA issuer
-        // The whole warp walks the schedule; lane 0 issues every MMA and every
-        // commit, so each commit covers all earlier MMAs.  Iteration q: the
-        // convs of quad q (pairs 2q, 2q+1), then dense-1 of quad q-1.
-        constexpr uint32_t idesc_conv = make_idesc(128, kPairN, FP16);
-        constexpr uint32_t idesc_fc1 = make_idesc(128, kN1, FP16);
-        const uint64_t convb_desc = sw128_desc(sConvB);
+    } else if (warp == 1 || warp == kFc1Warp) {
+        // ====================================================== MMA issuers
+        // Two warps issue MMAs, each walking its own schedule warp-wide with
+        // lane 0 issuing (so each commit covers all earlier MMAs of that
+        // thread): warp 1 the convs, pair by pair, as soon as an im2col tile
+        // and a free TMEM slot exist; warp kFc1Warp dense-1, pair by pair, as
+        // soon as the pair's activations and its W1 stage are in place.  The
+        // slot-free barrier (dense-1 done) orders a slot's reuse by the next
+        // conv; the activation barrier orders dense-1 after its conv.  Neither
+        // stream waits behind the other's dependencies.
+        const int np = 2 * nq;
         bool ok = true;
-        if (debug_stall) ok = warp_wait(bar(kBarStall), 0u, guard, lane);  // nothing arrives here
-        for (int q = 0; ok && q <= nq; ++q) {
-            if (q < nq) {
+        if (warp == 1) {
+            constexpr uint32_t idesc_conv = make_idesc(128, kPairN, FP16);
+            const uint64_t convb_desc = sw128_desc(sConvB);
+            if (debug_stall) ok = warp_wait(bar(kBarStall), 0u, guard, lane);  // nothing arrives here
+            for (int p = 0; ok && p < np; ++p) {
+                const int q = p >> 1, pr = p & 1;
                 const int ib = q % kImBufs;
-                if (!warp_wait(bar(kBarImFull + ib), (uint32_t)(q / kImBufs) & 1u, guard, lane)) {
+                const int s = p % kSlots;
+                if (pr == 0 && !warp_wait(bar(kBarImFull + ib), (uint32_t)(q / kImBufs) & 1u, guard, lane)) {
                     ok = false;
                     break;
                 }
-                for (int pr = 0; pr < 2; ++pr) {
-                    const int pi = 2 * q + pr;
-                    const int s = pi % kSlots;
-                    // the slot's previous pair (pi - kSlots) has been read by its dense-1
-                    if (pi >= kSlots &&
-                        !warp_wait(bar(kBarFree + s), (uint32_t)(pi / kSlots - 1) & 1u, guard, lane)) {
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
-                    if (lane == 0) {
-                        const uint32_t d = tmem + kSlotCol0 + (uint32_t)s * kSlotCols;
-                        const uint64_t ad = sw128_desc(sIm + ib * kImBytes) + (uint64_t)((pr * 64) >> 4);
-                        mma_ss(d, ad, convb_desc, idesc_conv, 0u);
-                        mma_ss(d, ad + (32u >> 4), convb_desc + (32u >> 4), idesc_conv, 1u);
-                        mma_commit(bar(kBarConv + s));
-                    }
-                    __syncwarp();
+                // the slot's previous pair (p - kSlots) has been read by its dense-1
+                if (p >= kSlots && !warp_wait(bar(kBarFree + s), (uint32_t)(p / kSlots - 1) & 1u, guard, lane)) {
+                    ok = false;
+                    break;
                 }
-                if (!ok) break;
-                if (lane == 0) mma_commit(bar(kBarImFree + ib));
+                tc_fence_after();
+                if (lane == 0) {
+                    const uint32_t d = tmem + kSlotCol0 + (uint32_t)s * kSlotCols;
+                    const uint64_t ad = sw128_desc(sIm + ib * kImBytes) + (uint64_t)((pr * 64) >> 4);
+                    mma_ss(d, ad, convb_desc, idesc_conv, 0u);
+                    mma_ss(d, ad + (32u >> 4), convb_desc + (32u >> 4), idesc_conv, 1u);
+                    mma_commit(bar(kBarConv + s));
+                    if (pr == 1) mma_commit(bar(kBarImFree + ib));
+                }
                 __syncwarp();
             }
-            const int qq = q - 1;
-            if (qq >= 0) {
-                const int wj = qq % kW1Stages;
-                if (!warp_wait(bar(kBarW1Full + wj), (uint32_t)(qq / kW1Stages) & 1u, guard, lane)) {
+        } else {
+            constexpr uint32_t idesc_fc1 = make_idesc(128, kN1, FP16);
+            for (int f = 0; ok && f < np; ++f) {
+                const int qf = f >> 1, pf = f & 1;
+                const int wj = qf % kW1Stages;
+                const int s = f % kSlots;
+                if (pf == 0 && !warp_wait(bar(kBarW1Full + wj), (uint32_t)(qf / kW1Stages) & 1u, guard, lane)) {
                     ok = false;
                     break;
                 }
-                const uint64_t wdesc = sw128_desc(sW1 + wj * kW1StageBytes);
-                for (int pr = 0; pr < 2; ++pr) {
-                    const int pi = 2 * qq + pr;
-                    const int s = pi % kSlots;
-                    if (!warp_wait(bar(kBarAct + s), (uint32_t)(pi / kSlots) & 1u, guard, lane)) {
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
-                    if (lane == 0) {
-                        const uint32_t a = tmem + kSlotCol0 + (uint32_t)s * kSlotCols;
+                if (!warp_wait(bar(kBarAct + s), (uint32_t)(f / kSlots) & 1u, guard, lane)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                if (lane == 0) {
+                    const uint64_t wdesc = sw128_desc(sW1 + wj * kW1StageBytes);
+                    const uint32_t a = tmem + kSlotCol0 + (uint32_t)s * kSlotCols;
 #pragma unroll
-                        for (int t = 0; t < 6; ++t) {
-                            const int step = pr * 6 + t;  // 16-wide K step inside the quad's 192
-                            const uint64_t bd =
-                                wdesc + (uint64_t)(((step >> 2) * kW1BoxBytes + (step & 3) * 32) >> 4);
-                            mma_ts(tmem + kAccCol, a + 8u * t, bd, idesc_fc1, (qq > 0 || step > 0) ? 1u : 0u);
-                        }
-                        mma_commit(bar(kBarFree + s));
+                    for (int t = 0; t < 6; ++t) {
+                        const int step = pf * 6 + t;  // 16-wide K step inside the quad's 192
+                        const uint64_t bd = wdesc + (uint64_t)(((step >> 2) * kW1BoxBytes + (step & 3) * 32) >> 4);
+                        mma_ts(tmem + kAccCol, a + 8u * t, bd, idesc_fc1, (f > 0 || t > 0) ? 1u : 0u);
                     }
-                    __syncwarp();
+                    mma_commit(bar(kBarFree + s));
+                    if (pf == 1) mma_commit(bar(kBarW1Empty + wj));
                 }
-                if (!ok) break;
-                if (lane == 0) mma_commit(bar(kBarW1Empty + wj));
                 __syncwarp();
             }
+            if (lane == 0 && ok) mma_commit(bar(kBarAcc));
         }
         if (lane == 0) {
-            if (ok) mma_commit(bar(kBarAcc));
-            // every MMA issued so far completes before TMEM is released
+            // every MMA either warp issued completes before TMEM is released:
+            // the drain barrier expects one commit from each issuer
             mma_commit(bar(kBarDrain));
             const uint64_t t0 = global_timer_ns();
             while (!mbar_try_wait(bar(kBarDrain), 0u) && (int64_t)(global_timer_ns() - t0) < (int64_t)timeout_ns) {
@@ -492,7 +490,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 if (lane == 0) mbar_arrive(bar(kBarImFull + ib));
             }
         }
-    } else {
+    } else if (warp < kFc1Warp) {
         // ================================== conv epilogue + dense-1 store
         const int q4 = warp & 3;
         const int row = 32 * q4 + lane;
