@@ -346,77 +346,74 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         }
     } else if (warp == 1 || warp == kFc1Warp) {
         // ====================================================== MMA issuers
-        // Two warps issue MMAs, each walking its own schedule warp-wide with
-        // lane 0 issuing (so each commit covers all earlier MMAs of that
-        // thread): warp 1 the convs, pair by pair, as soon as an im2col tile
-        // and a free TMEM slot exist; warp kFc1Warp dense-1, pair by pair, as
-        // soon as the pair's activations and its W1 stage are in place.  The
-        // slot-free barrier (dense-1 done) orders a slot's reuse by the next
-        // conv; the activation barrier orders dense-1 after its conv.  Neither
-        // stream waits behind the other's dependencies.
-        const int np = 2 * nq;
-        bool ok = true;
-        if (warp == 1) {
-            constexpr uint32_t idesc_conv = make_idesc(128, kPairN, FP16);
-            const uint64_t convb_desc = sw128_desc(sConvB);
-            if (debug_stall) ok = warp_wait(bar(kBarStall), 0u, guard, lane);  // nothing arrives here
-            for (int p = 0; ok && p < np; ++p) {
-                const int q = p >> 1, pr = p & 1;
-                const int ib = q % kImBufs;
-                const int s = p % kSlots;
-                if (pr == 0 && !warp_wait(bar(kBarImFull + ib), (uint32_t)(q / kImBufs) & 1u, guard, lane)) {
-                    ok = false;
-                    break;
-                }
-                // the slot's previous pair (p - kSlots) has been read by its dense-1
-                if (p >= kSlots && !warp_wait(bar(kBarFree + s), (uint32_t)(p / kSlots - 1) & 1u, guard, lane)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                if (lane == 0) {
-                    const uint32_t d = tmem + kSlotCol0 + (uint32_t)s * kSlotCols;
-                    const uint64_t ad = sw128_desc(sIm + ib * kImBytes) + (uint64_t)((pr * 64) >> 4);
-                    mma_ss(d, ad, convb_desc, idesc_conv, 0u);
-                    mma_ss(d, ad + (32u >> 4), convb_desc + (32u >> 4), idesc_conv, 1u);
-                    mma_commit(bar(kBarConv + s));
-                    if (pr == 1) mma_commit(bar(kBarImFree + ib));
-                }
-                __syncwarp();
-            }
-        } else {
-            constexpr uint32_t idesc_fc1 = make_idesc(128, kN1, FP16);
-            for (int f = 0; ok && f < np; ++f) {
-                const int qf = f >> 1, pf = f & 1;
-                const int wj = qf % kW1Stages;
-                const int s = f % kSlots;
-                if (pf == 0 && !warp_wait(bar(kBarW1Full + wj), (uint32_t)(qf / kW1Stages) & 1u, guard, lane)) {
-                    ok = false;
-                    break;
-                }
-                if (!warp_wait(bar(kBarAct + s), (uint32_t)(f / kSlots) & 1u, guard, lane)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                if (lane == 0) {
-                    const uint64_t wdesc = sw128_desc(sW1 + wj * kW1StageBytes);
-                    const uint32_t a = tmem + kSlotCol0 + (uint32_t)s * kSlotCols;
-#pragma unroll
-                    for (int t = 0; t < 6; ++t) {
-                        const int step = pf * 6 + t;  // 16-wide K step inside the quad's 192
-                        const uint64_t bd = wdesc + (uint64_t)(((step >> 2) * kW1BoxBytes + (step & 3) * 32) >> 4);
-                        mma_ts(tmem + kAccCol, a + 8u * t, bd, idesc_fc1, (f > 0 || t > 0) ? 1u : 0u);
-                    }
-                    mma_commit(bar(kBarFree + s));
-                    if (pf == 1) mma_commit(bar(kBarW1Empty + wj));
-                }
-                __syncwarp();
-            }
-            if (lane == 0 && ok) mma_commit(bar(kBarAcc));
-        }
+        // Two threads issue MMAs, lane 0 of warp 1 (the convs) and lane 0 of
+        // warp kFc1Warp (dense-1); each walks its own schedule alone, so that
+        // nothing but its waits stands between its groups of MMAs (the tensor
+        // pipe's queue is shallow: an issuing thread runs at the pace of
+        // execution).  The conv thread issues a pair as soon as its im2col
+        // tile and a free TMEM slot exist; the dense-1 thread issues a quad
+        // (12 MMAs into the accumulator, the first pair's slot freed after
+        // its 6) as soon as both pairs' activations and the W1 stage are in.
+        // The slot-free barrier orders a slot's reuse after its dense-1; the
+        // activation barrier orders dense-1 after its conv.  Each commit covers
+        // all earlier MMAs of its thread.
         if (lane == 0) {
-            // every MMA either warp issued completes before TMEM is released:
+            bool ok = true;
+            if (warp == 1) {
+                constexpr uint32_t idesc_conv = make_idesc(128, kPairN, FP16);
+                const uint64_t convb_desc = sw128_desc(sConvB);
+                if (debug_stall) ok = wait_bounded(bar(kBarStall), 0u, guard);  // nothing arrives here
+                for (int q = 0; ok && q < nq; ++q) {
+                    const int ib = q % kImBufs;
+                    if (!wait_bounded(bar(kBarImFull + ib), (uint32_t)(q / kImBufs) & 1u, guard)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint64_t im_desc = sw128_desc(sIm + ib * kImBytes);
+                    for (int pr = 0; pr < 2; ++pr) {
+                        const int p = 2 * q + pr;
+                        const int s = p % kSlots;
+                        // the slot's previous pair (p - kSlots) has been read by its dense-1
+                        if (p >= kSlots && !wait_bounded(bar(kBarFree + s), (uint32_t)(p / kSlots - 1) & 1u, guard)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint32_t d = tmem + kSlotCol0 + (uint32_t)s * kSlotCols;
+                        const uint64_t ad = im_desc + (uint64_t)((pr * 64) >> 4);
+                        mma_ss(d, ad, convb_desc, idesc_conv, 0u);
+                        mma_ss(d, ad + (32u >> 4), convb_desc + (32u >> 4), idesc_conv, 1u);
+                        mma_commit(bar(kBarConv + s));
+                    }
+                    if (!ok) break;
+                    mma_commit(bar(kBarImFree + ib));
+                }
+            } else {
+                constexpr uint32_t idesc_fc1 = make_idesc(128, kN1, FP16);
+                for (int q = 0; ok && q < nq; ++q) {
+                    const int wj = q % kW1Stages;
+                    const int s0 = (2 * q) % kSlots, s1 = (2 * q + 1) % kSlots;
+                    const uint32_t par = (uint32_t)((2 * q) / kSlots) & 1u;  // same use for both slots
+                    if (!wait_bounded(bar(kBarW1Full + wj), (uint32_t)(q / kW1Stages) & 1u, guard) ||
+                        !wait_bounded(bar(kBarAct + s0), par, guard) || !wait_bounded(bar(kBarAct + s1), par, guard)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint64_t wdesc = sw128_desc(sW1 + wj * kW1StageBytes);
+#pragma unroll
+                    for (int step = 0; step < 12; ++step) {  // 16-wide K steps of the quad's 192
+                        const uint32_t a = tmem + kSlotCol0 + (uint32_t)(step < 6 ? s0 : s1) * kSlotCols + 8u * (step % 6);
+                        const uint64_t bd = wdesc + (uint64_t)(((step >> 2) * kW1BoxBytes + (step & 3) * 32) >> 4);
+                        mma_ts(tmem + kAccCol, a, bd, idesc_fc1, (q > 0 || step > 0) ? 1u : 0u);
+                        if (step == 5) mma_commit(bar(kBarFree + s0));
+                    }
+                    mma_commit(bar(kBarFree + s1));
+                    mma_commit(bar(kBarW1Empty + wj));
+                }
+                if (ok) mma_commit(bar(kBarAcc));
+            }
+            // every MMA either thread issued completes before TMEM is released:
             // the drain barrier expects one commit from each issuer
             mma_commit(bar(kBarDrain));
             const uint64_t t0 = global_timer_ns();
