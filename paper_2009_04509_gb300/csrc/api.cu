@@ -151,11 +151,13 @@ emtk_status run_network(emtk_ctx *c, const void *patches, int32_t n, float *cons
     const int n_pad = n_pad_of(n);
     const int max_splits = (int)std::max<int64_t>(1, kPartialCap / ((int64_t)n_pad * kN1));
     cudaError_t e;
-    int splits;
+    int splits = 0, G = 0;
     if (tensor_precision(c->opt.precision)) {
-        splits = choose_splits_tc(n, c->sm_count, max_splits);
+        // one persistent CTA per SM (stream-K), fewer if the partial rows would not fit
+        G = c->sm_count;
+        while (G > 1 && streamk_partial_rows(n, G) > max_splits) G /= 2;
         Prof prof(c, EMTK_KERNEL_NETWORK, s);
-        e = launch_cnn_tc(c->w, patches, c->opt.precision == EMTK_FP16, n, splits, c->ws.partials, n_pad,
+        e = launch_cnn_tc(c->w, patches, c->opt.precision == EMTK_FP16, n, G, c->ws.partials, n_pad,
                           c->ws.status, c->opt.wait_timeout_ns, c->opt.debug_stall, s);
     } else {
         splits = choose_splits_fp32(n, c->sm_count, max_splits);
@@ -165,7 +167,7 @@ emtk_status run_network(emtk_ctx *c, const void *patches, int32_t n, float *cons
     if (e != cudaSuccess) return cuda_status(e);
     {
         Prof prof(c, EMTK_KERNEL_HEAD, s);
-        e = launch_head(c->w, c->ws.partials, splits, n_pad, n, dest, c->opt.debug_logits, s);
+        e = launch_head(c->w, c->ws.partials, splits, G, n_pad, n, dest, c->opt.debug_logits, s);
     }
     count_launch(c, n);
     return cuda_status(e);

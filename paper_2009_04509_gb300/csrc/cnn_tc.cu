@@ -42,7 +42,7 @@ constexpr int kW1Stages = 3;     // shared-memory stages of W1 (one quad each)
 constexpr int kImBufs = 3;       // shared-memory im2col tiles (one quad each)
 constexpr int kSlots = 4;        // TMEM conv/activation slots (one pair each)
 constexpr int kPosPerW1 = 4;     // conv positions per W1 stage = per quad
-constexpr int kW1Steps = kPos / kPosPerW1;                  // 484 quads
+constexpr int kW1Steps = kQuads;                             // 484 quads
 constexpr int kW1Box = 64;                                   // K elements per TMA box (128 B)
 constexpr int kW1BoxBytes = kW1Box * kN1 * 2;                // 16384
 constexpr int kBoxesPerStage = kPosPerW1 * kF / kW1Box;      // 3
@@ -69,8 +69,9 @@ constexpr int kBarImFree = kBarImFull + kImBufs;     // im2col tile read by its 
 constexpr int kBarConv = kBarImFree + kImBufs;       // conv tile of a pair done (MMA commit)
 constexpr int kBarAct = kBarConv + kSlots;           // activations written (4 epilogue warps)
 constexpr int kBarFree = kBarAct + kSlots;           // dense-1 of the slot's pair done (MMA commit)
-constexpr int kBarAcc = kBarFree + kSlots;
-constexpr int kBarStall = kBarAcc + 1;
+constexpr int kBarAcc = kBarFree + kSlots;             // a tile's dense-1 done (MMA commit)
+constexpr int kBarAccEmpty = kBarAcc + 1;             // accumulator drained (4 epilogue warps)
+constexpr int kBarStall = kBarAccEmpty + 1;
 constexpr int kBarDrain = kBarStall + 1;
 constexpr int kNumBars = kBarDrain + 1;
 constexpr int kOffTmemSlot = kOffBar + kNumBars * 8;
@@ -250,7 +251,7 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
 template <bool FP16>
 __global__ void __launch_bounds__(kThreadsTC, 1)
     cnn_tc_kernel(const __grid_constant__ CUtensorMap tmap_w1, const uint16_t *__restrict__ patches, int n,
-                  const uint16_t *__restrict__ convB_g, float *__restrict__ partials, int n_pad, int splits,
+                  const uint16_t *__restrict__ convB_g, float *__restrict__ partials, int n_pad, long long units,
                   int *status, long long timeout_ns, int debug_stall) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_u32 = smem_u32(smem_raw);
@@ -265,11 +266,13 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const int m_tile = blockIdx.x;
-    const int seg = blockIdx.y;
-    const int j0 = (int)((int64_t)seg * kW1Steps / splits);   // first quad
-    const int j1 = (int)((int64_t)(seg + 1) * kW1Steps / splits);
-    const int nq = j1 - j0;                                     // quads in this segment
+    const int cta = blockIdx.x;
+    const int G = gridDim.x;
+    const int64_t u0 = unit_begin(cta, units, G);   // this CTA's units [u0, u1)
+    const int64_t u1 = unit_begin(cta + 1, units, G);
+    const int nq = (int)(u1 - u0);                  // quads, in order, across tile boundaries
+    const int qt0 = (int)(u0 % kW1Steps);           // quad-in-tile and tile of the first unit
+    const int tile0 = (int)(u0 / kW1Steps);
     const Guard guard{abort_flag, status, (int64_t)timeout_ns};
 
     // ---- set-up: pair conv B operand into swizzled smem, barriers, TMEM
@@ -294,6 +297,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
             mbar_init(bar(kBarFree + i), 1);
         }
         mbar_init(bar(kBarAcc), 1);
+        mbar_init(bar(kBarAccEmpty), 4);
         mbar_init(bar(kBarStall), 1);
         mbar_init(bar(kBarDrain), 2);
         *abort_flag = 0u;
@@ -316,7 +320,8 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         if (lane == 0) {
             int issued = 0;
             bool ok = true;
-            for (int jj = 0; jj < nq; ++jj) {
+            int qt = qt0;
+            for (int jj = 0; jj < nq; ++jj, qt = (qt + 1 == kW1Steps) ? 0 : qt + 1) {
                 const int wj = jj % kW1Stages;
                 const uint32_t use = (uint32_t)(jj / kW1Stages);
                 if (jj >= kW1Stages && !wait_bounded(bar(kBarW1Empty + wj), (use - 1u) & 1u, guard)) {
@@ -331,7 +336,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
 #pragma unroll
                 for (int a = 0; a < kBoxesPerStage; ++a)
                     tma_load_3d(sW1 + wj * kW1StageBytes + a * kW1BoxBytes, &tmap_w1, bar(kBarW1Full + wj), 0, 0,
-                                kBoxesPerStage * (j0 + jj) + a);
+                                kBoxesPerStage * qt + a);
                 ++issued;
             }
             if (!ok) {  // let copies in flight land before the CTA's memory goes away
@@ -390,12 +395,23 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 }
             } else {
                 constexpr uint32_t idesc_fc1 = make_idesc(128, kN1, FP16);
+                int tiles_done = 0;  // tile segments whose accumulator was handed to the epilogue
+                int qt = qt0 - 1;
                 for (int q = 0; ok && q < nq; ++q) {
+                    qt = (qt + 1 == kW1Steps) ? 0 : qt + 1;
+                    const bool first = (q == 0) || (qt == 0);
+                    const bool last = (q == nq - 1) || (qt == kW1Steps - 1);
                     const int wj = q % kW1Stages;
                     const int s0 = (2 * q) % kSlots, s1 = (2 * q + 1) % kSlots;
                     const uint32_t par = (uint32_t)((2 * q) / kSlots) & 1u;  // same use for both slots
                     if (!wait_bounded(bar(kBarW1Full + wj), (uint32_t)(q / kW1Stages) & 1u, guard) ||
                         !wait_bounded(bar(kBarAct + s0), par, guard) || !wait_bounded(bar(kBarAct + s1), par, guard)) {
+                        ok = false;
+                        break;
+                    }
+                    // a new tile starts from zero in the accumulator, once the epilogue drained the last one
+                    if (first && tiles_done > 0 &&
+                        !wait_bounded(bar(kBarAccEmpty), (uint32_t)(tiles_done - 1) & 1u, guard)) {
                         ok = false;
                         break;
                     }
@@ -405,13 +421,16 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                     for (int step = 0; step < 12; ++step) {  // 16-wide K steps of the quad's 192
                         const uint32_t a = tmem + kSlotCol0 + (uint32_t)(step < 6 ? s0 : s1) * kSlotCols + 8u * (step % 6);
                         const uint64_t bd = wdesc + (uint64_t)(((step >> 2) * kW1BoxBytes + (step & 3) * 32) >> 4);
-                        mma_ts(tmem + kAccCol, a, bd, idesc_fc1, (q > 0 || step > 0) ? 1u : 0u);
+                        mma_ts(tmem + kAccCol, a, bd, idesc_fc1, (first && step == 0) ? 0u : 1u);
                         if (step == 5) mma_commit(bar(kBarFree + s0));
                     }
                     mma_commit(bar(kBarFree + s1));
                     mma_commit(bar(kBarW1Empty + wj));
+                    if (last) {
+                        mma_commit(bar(kBarAcc));
+                        ++tiles_done;
+                    }
                 }
-                if (ok) mma_commit(bar(kBarAcc));
             }
             // every MMA either thread issued completes before TMEM is released:
             // the drain barrier expects one commit from each issuer
@@ -430,17 +449,21 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         // even, taps (2k, 2k+1) are one aligned pixel pair of the patch row.
         const int q4 = warp & 3;
         const int row = 32 * q4 + lane;
-        const int64_t hit = (int64_t)m_tile * 128 + row;
-        const bool valid = hit < n;
-        const uint4 *prow = reinterpret_cast<const uint4 *>(patches) + (valid ? hit : 0) * (kPatchElems / 8);
         const uint32_t one = FP16 ? 0x3C00u : 0x3F80u;
         const uint32_t ones = one | (one << 16);
         uint8_t *my_row = gbase + kOffIm + row * 128;
-        const int p0 = j0 * kPosPerW1;
-        const int p1 = j1 * kPosPerW1;
-        const int y_first = p0 / kQ;
-        const int y_last = nq > 0 ? (p1 - 1) / kQ : y_first - 1;
         bool ok = true;
+        const int t_first = tile0;
+        const int t_last = nq > 0 ? (int)((u1 - 1) / kW1Steps) : t_first - 1;
+        for (int tile = t_first; ok && tile <= t_last; ++tile) {
+        const int j0 = tile == t_first ? qt0 : 0;   // quads of this tile in [j0, j1)
+        const int j1 = tile == t_last ? (int)((u1 - 1) % kW1Steps) + 1 : kW1Steps;
+        const int64_t k_base = (int64_t)tile * kW1Steps - u0;        // running quad index = k_base + quad
+        const int64_t hit = (int64_t)tile * 128 + row;
+        const bool valid = hit < n;
+        const uint4 *prow = reinterpret_cast<const uint4 *>(patches) + (valid ? hit : 0) * (kPatchElems / 8);
+        const int y_first = j0 * kPosPerW1 / kQ;
+        const int y_last = (j1 * kPosPerW1 - 1) / kQ;
         for (int y = y_first; ok && y <= y_last; ++y) {
             uint32_t R[kK][24];  // patch rows y..y+4 of this hit, 2 pixels per word
 #pragma unroll
@@ -458,7 +481,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
             for (int xq = 0; xq < kQ / kPosPerW1; ++xq) {
                 const int quad = (y * kQ) / kPosPerW1 + xq;
                 if (quad < j0 || quad >= j1) continue;
-                const int k = quad - j0;
+                const int k = (int)(k_base + quad);
                 const int ib = k % kImBufs;
                 if (k >= kImBufs &&
                     !warp_wait(bar(kBarImFree + ib), (uint32_t)(k / kImBufs - 1) & 1u, guard, lane)) {
@@ -487,13 +510,15 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 if (lane == 0) mbar_arrive(bar(kBarImFull + ib));
             }
         }
+        }
     } else if (warp < kFc1Warp) {
         // ================================== conv epilogue + dense-1 store
         const int q4 = warp & 3;
         const int row = 32 * q4 + lane;
-        const int64_t hit = (int64_t)m_tile * 128 + row;
         const uint32_t lane_tmem = tmem + ((uint32_t)(32 * q4) << 16);
         bool ok = true;
+        int tiles_done = 0;
+        int qt = qt0;       // quad-in-tile of pair pi
         for (int pi = 0; pi < 2 * nq; ++pi) {
             const int s = pi % kSlots;
             if (!warp_wait(bar(kBarConv + s), (uint32_t)(pi / kSlots) & 1u, guard, lane)) {
@@ -520,26 +545,41 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(bar(kBarAct + s));
-        }
-        if (ok && nq > 0 && warp_wait(bar(kBarAcc), 0u, guard, lane)) {
-            tc_fence_after();
-            float *dst = partials + ((int64_t)seg * n_pad + hit) * kN1;
-#pragma unroll
-            for (int c = 0; c < kN1 / 32; ++c) {
-                uint32_t r[32];
-                tmem_ld16<0>(lane_tmem + kAccCol + 32u * c, r);
-                tmem_ld16<16>(lane_tmem + kAccCol + 32u * c + 16u, r);
-                tmem_ld_wait();
-                reg_fence(r);
-                if (hit < n) {
-#pragma unroll
-                    for (int e = 0; e < 8; ++e)
-                        reinterpret_cast<float4 *>(dst + 32 * c)[e] =
-                            make_float4(__uint_as_float(r[4 * e]), __uint_as_float(r[4 * e + 1]),
-                                        __uint_as_float(r[4 * e + 2]), __uint_as_float(r[4 * e + 3]));
+            // after a tile's last pair: drain its dense-1 accumulator to the partial-sum row
+            const bool tile_end = (pi & 1) && ((pi >> 1) == nq - 1 || qt == kW1Steps - 1);
+            if (pi & 1) qt = (qt + 1 == kW1Steps) ? 0 : qt + 1;
+            if (tile_end) {
+                if (!warp_wait(bar(kBarAcc), (uint32_t)tiles_done & 1u, guard, lane)) {
+                    ok = false;
+                    break;
                 }
+                tc_fence_after();
+                const int64_t tile = tile0 + tiles_done;
+                const int krow = cta - cta_of_unit(tile * kW1Steps, units, G);
+                const int64_t hit = tile * 128 + row;
+                float *dst = partials + ((int64_t)krow * n_pad + hit) * kN1;
+#pragma unroll
+                for (int c = 0; c < kN1 / 32; ++c) {
+                    uint32_t r[32];
+                    tmem_ld16<0>(lane_tmem + kAccCol + 32u * c, r);
+                    tmem_ld16<16>(lane_tmem + kAccCol + 32u * c + 16u, r);
+                    tmem_ld_wait();
+                    reg_fence(r);
+                    if (hit < n) {
+#pragma unroll
+                        for (int e = 0; e < 8; ++e)
+                            reinterpret_cast<float4 *>(dst + 32 * c)[e] =
+                                make_float4(__uint_as_float(r[4 * e]), __uint_as_float(r[4 * e + 1]),
+                                            __uint_as_float(r[4 * e + 2]), __uint_as_float(r[4 * e + 3]));
+                    }
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar(kBarAccEmpty));
+                ++tiles_done;
             }
         }
+        (void)ok;
     }
 
     tc_fence_before();
@@ -635,39 +675,34 @@ cudaError_t prepare_tc_weights(DeviceWeights &w, const emtk_weights &hw, bool fp
     return cudaSuccess;
 }
 
-// Splits of the dense-1 input (in quads) so that m_tiles x splits CTAs fill
-// the SMs in few, even waves.  Time model per wave: the segment's quads plus
-// a fixed cost of about 6 quads (pipeline fill and drain, partial-sum store).
-int choose_splits_tc(int n, int sm_count, int max_splits) {
+// Partial-sum rows a stream-K launch over G CTAs needs: the largest number
+// of CTAs that share one tile.
+int streamk_partial_rows(int32_t n, int G) {
     const int m_tiles = (n + 127) / 128;
-    int best = 1;
-    double best_t = 1e30;
-    const int cap = max_splits < kW1Steps / 4 ? max_splits : kW1Steps / 4;
-    for (int s = 1; s <= cap; ++s) {
-        const int64_t ctas = (int64_t)m_tiles * s;
-        const int64_t waves = (ctas + sm_count - 1) / sm_count;
-        const double t = (double)waves * ((double)kW1Steps / s + 6.0);
-        if (t < best_t - 1e-9) {
-            best_t = t;
-            best = s;
-        }
+    const int64_t units = (int64_t)m_tiles * kW1Steps;
+    int rows = 1;
+    for (int t = 0; t < m_tiles; ++t) {
+        const int a = cta_of_unit((int64_t)t * kW1Steps, units, G);
+        const int b = cta_of_unit((int64_t)t * kW1Steps + kW1Steps - 1, units, G);
+        rows = b - a + 1 > rows ? b - a + 1 : rows;
     }
-    return best;
+    return rows;
 }
 
-cudaError_t launch_cnn_tc(const DeviceWeights &w, const void *patches, bool fp16, int32_t n, int splits,
+cudaError_t launch_cnn_tc(const DeviceWeights &w, const void *patches, bool fp16, int32_t n, int G,
                           float *partials, int n_pad, int *status, int64_t timeout_ns, int debug_stall,
                           cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
     const CUtensorMap &map = *static_cast<const CUtensorMap *>(w.w1_tmap);
-    dim3 grid((n + 127) / 128, splits);
+    const long long units = (long long)((n + 127) / 128) * kW1Steps;
+    dim3 grid(G);
     if (fp16)
         cnn_tc_kernel<true><<<grid, kThreadsTC, kSmemBytesTC, s>>>(map, static_cast<const uint16_t *>(patches), n,
-                                                                   w.convB, partials, n_pad, splits, status,
+                                                                   w.convB, partials, n_pad, units, status,
                                                                    (long long)timeout_ns, debug_stall);
     else
         cnn_tc_kernel<false><<<grid, kThreadsTC, kSmemBytesTC, s>>>(map, static_cast<const uint16_t *>(patches), n,
-                                                                    w.convB, partials, n_pad, splits, status,
+                                                                    w.convB, partials, n_pad, units, status,
                                                                     (long long)timeout_ns, debug_stall);
     return cudaGetLastError();
 }

@@ -23,6 +23,20 @@ constexpr int kN1 = 128;
 constexpr int kN2 = 32;
 constexpr int kNC = 3;
 constexpr int kPatchElems = kPatch * kPatch;         // 2304
+constexpr int kQuads = kPos / 4;                     // 484 quads of 4 conv positions
+
+// Stream-K split of the tensor-core network: the launch's work is the units
+// u = tile * kQuads + quad (tile = 128 hits); CTA c of G takes the contiguous
+// units [unit_begin(c), unit_begin(c + 1)).  A tile's dense-1 partial sums
+// come from CTAs cta_of_unit(first unit) .. cta_of_unit(last unit), written
+// to partial rows 0, 1, ... in that order.
+__host__ __device__ inline int64_t unit_begin(int c, int64_t units, int G) { return (int64_t)c * units / G; }
+__host__ __device__ inline int cta_of_unit(int64_t u, int64_t units, int G) {
+    int c = (int)((u * G) / units);
+    while (c > 0 && unit_begin(c, units, G) > u) --c;
+    while (c + 1 < G && unit_begin(c + 1, units, G) <= u) ++c;
+    return c;
+}
 
 // Requests handled by one extraction launch (kernel-parameter table).
 constexpr int kMaxReqPerLaunch = 64;
@@ -112,11 +126,16 @@ cudaError_t launch_fill_dest(float *scores, int out_stride, float **dest, int32_
 // Network: dense-1 partial sums [splits][n_pad][128] from patches.
 cudaError_t launch_cnn_fp32(const DeviceWeights &w, const float *patches, int32_t n, int splits,
                             float *partials, int n_pad, cudaStream_t s);
-cudaError_t launch_cnn_tc(const DeviceWeights &w, const void *patches, bool fp16, int32_t n,
-                          int splits, float *partials, int n_pad, int *status, int64_t timeout_ns,
-                          int debug_stall, cudaStream_t s);
-// Sum of partials + bias + ReLU, dense-2, heads; scores to dest[h].
-cudaError_t launch_head(const DeviceWeights &w, const float *partials, int splits, int n_pad,
+// Stream-K over G CTAs (one per SM); partials [rows][n_pad][128] with rows
+// = streamk_partial_rows(n, G).
+cudaError_t launch_cnn_tc(const DeviceWeights &w, const void *patches, bool fp16, int32_t n, int G,
+                          float *partials, int n_pad, int *status, int64_t timeout_ns, int debug_stall,
+                          cudaStream_t s);
+int streamk_partial_rows(int32_t n, int G);
+// Sum of partials + bias + ReLU, dense-2, heads; scores to dest[h].  Partial
+// rows: `splits` per hit (G == 0), or the stream-K contributors of the hit's
+// tile (G > 0).
+cudaError_t launch_head(const DeviceWeights &w, const float *partials, int splits, int G, int n_pad,
                         int32_t n, float *const *dest, int debug_logits, cudaStream_t s);
 
 // Kernel attributes (dynamic shared memory), set once per device at create.
@@ -125,7 +144,6 @@ cudaError_t init_tc_kernel_attrs();
 
 // Host helpers for the tensor-core weights (cnn_tc.cu).
 cudaError_t prepare_tc_weights(DeviceWeights &w, const emtk_weights &hw, bool fp16);
-int choose_splits_tc(int n, int sm_count, int max_splits);
 int choose_splits_fp32(int n, int sm_count, int max_splits);
 
 }  // namespace emtk

@@ -1,15 +1,17 @@
-// Network tail (Sec. 2.2), fp32: sum of the dense-1 segment partials in
-// segment order + bias + ReLU, dense 128->32 + ReLU, the 3-way softmax head
-// (track, em, none) and the Michel sigmoid head.  One warp per hit; lane l
-// owns dense-1 outputs 4l..4l+3 and dense-2 output l.
+// Network tail (Sec. 2.2), fp32: sum of the dense-1 partial-sum rows in row
+// order + bias + ReLU, dense 128->32 + ReLU, the 3-way softmax head (track,
+// em, none) and the Michel sigmoid head.  One warp per hit; lane l owns
+// dense-1 outputs 4l..4l+3 and dense-2 output l.  The rows of a hit are the
+// K-splits of the fp32 path, or the stream-K CTAs that shared its tile.
 #include "emtk_internal.h"
 
 namespace emtk {
 namespace {
 
 constexpr int kWarps = 8;
+constexpr int kHitsPerWarp = 8;  // each block stages the tail weights once for 64 hits
 
-__global__ void __launch_bounds__(kWarps * 32) head_kernel(const float *__restrict__ partials, int splits, int n_pad,
+__global__ void __launch_bounds__(kWarps * 32) head_kernel(const float *__restrict__ partials, int splits, int G, int n_pad,
                                                           int32_t n, const float *__restrict__ fc1_b,
                                                           const float *__restrict__ fc2_w,
                                                           const float *__restrict__ fc2_b,
@@ -26,11 +28,18 @@ __global__ void __launch_bounds__(kWarps * 32) head_kernel(const float *__restri
     __syncthreads();
 
     const int lane = threadIdx.x & 31;
-    const int64_t h = (int64_t)blockIdx.x * kWarps + (threadIdx.x >> 5);
+    for (int j = 0; j < kHitsPerWarp; ++j) {
+    const int64_t h = ((int64_t)blockIdx.x * kWarps + (threadIdx.x >> 5)) * kHitsPerWarp + j;
     if (h >= n) return;
 
+    int rows = splits;
+    if (G > 0) {
+        const int64_t units = (int64_t)((n + 127) / 128) * kQuads;
+        const int64_t tile = h >> 7;
+        rows = cta_of_unit(tile * kQuads + kQuads - 1, units, G) - cta_of_unit(tile * kQuads, units, G) + 1;
+    }
     float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int s = 0; s < splits; ++s) {
+    for (int s = 0; s < rows; ++s) {
         const float4 v = __ldcs(reinterpret_cast<const float4 *>(partials + ((int64_t)s * n_pad + h) * kN1) + lane);
         a.x += v.x;
         a.y += v.y;
@@ -77,14 +86,16 @@ __global__ void __launch_bounds__(kWarps * 32) head_kernel(const float *__restri
             out[7] = z[3];
         }
     }
+    }
 }
 
 }  // namespace
 
-cudaError_t launch_head(const DeviceWeights &w, const float *partials, int splits, int n_pad, int32_t n,
+cudaError_t launch_head(const DeviceWeights &w, const float *partials, int splits, int G, int n_pad, int32_t n,
                         float *const *dest, int debug_logits, cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
-    head_kernel<<<(n + kWarps - 1) / kWarps, kWarps * 32, 0, s>>>(partials, splits, n_pad, n, w.fc1_b, w.fc2_w,
+    const int per_block = kWarps * kHitsPerWarp;
+    head_kernel<<<(n + per_block - 1) / per_block, kWarps * 32, 0, s>>>(partials, splits, G, n_pad, n, w.fc1_b, w.fc2_w,
                                                                   w.fc2_b, w.cls_w, w.cls_b, w.mic_w, w.mic_b,
                                                                   dest, debug_logits);
     return cudaGetLastError();
