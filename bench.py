@@ -204,10 +204,19 @@ def main():
     for _ in range(args.warmup):
         step()
     assert emtk.emtk_check(ctx, stream) == emtk.EMTK_OK
-    base = emtk.emtk_get_stats(ctx)
 
+    # clocks are sampled every 200 ms from here to the end of the timed
+    # region; untimed steps keep the GPU under the same load for at least a
+    # second before it starts, so that the samples see the step's clocks
     clocks = ClockSampler(gpu_uuid())
     clocks.start()
+    t_soak = time.perf_counter()
+    while time.perf_counter() - t_soak < 1.0:
+        for _ in range(10):
+            step()
+        torch.cuda.synchronize()
+    assert emtk.emtk_check(ctx, stream) == emtk.EMTK_OK
+    base = emtk.emtk_get_stats(ctx)
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     if dist:
         dist.barrier()
