@@ -63,7 +63,7 @@ void free_ctx(emtk_ctx *c) {
     for (void *p : {(void *)w.conv_w, (void *)w.conv_b, (void *)w.fc1_w, (void *)w.fc1_b, (void *)w.fc2_w,
                     (void *)w.fc2_b, (void *)w.cls_w, (void *)w.cls_b, (void *)w.mic_w, (void *)w.mic_b,
                     (void *)w.w1_tiles, (void *)w.convB, c->ws.dimg, c->ws.patches, (void *)c->ws.dest,
-                    (void *)c->ws.partials, (void *)c->ws.status})
+                    (void *)c->ws.partials, (void *)c->ws.status, (void *)c->ws.hdesc})
         if (p) cudaFree(p);
     delete static_cast<CUtensorMap *>(w.w1_tmap);
     delete c;
@@ -146,7 +146,10 @@ emtk_status ensure_dimg(emtk_ctx *c, size_t bytes, cudaStream_t s) {
 }
 
 // Network on `n` patches already in the workspace format -> scores via dest.
-emtk_status run_network(emtk_ctx *c, const void *patches, int32_t n, float *const *dest, cudaStream_t s) {
+// `desc` (tensor-core path only) locates each hit's window in the haloed
+// interval images at `patches`; without it `patches` holds the patches.
+emtk_status run_network(emtk_ctx *c, const void *patches, const HitDesc *desc, int32_t n, float *const *dest,
+                        cudaStream_t s) {
     if (n <= 0) return EMTK_OK;
     const int n_pad = n_pad_of(n);
     const int max_splits = (int)std::max<int64_t>(1, kPartialCap / ((int64_t)n_pad * kN1));
@@ -157,7 +160,7 @@ emtk_status run_network(emtk_ctx *c, const void *patches, int32_t n, float *cons
         G = c->sm_count;
         while (G > 1 && streamk_partial_rows(n, G) > max_splits) G /= 2;
         Prof prof(c, EMTK_KERNEL_NETWORK, s);
-        e = launch_cnn_tc(c->w, patches, c->opt.precision == EMTK_FP16, n, G, c->ws.partials, n_pad,
+        e = launch_cnn_tc(c->w, patches, desc, c->opt.precision == EMTK_FP16, n, G, c->ws.partials, n_pad,
                           c->ws.status, c->opt.wait_timeout_ns, c->opt.debug_stall, s);
     } else {
         splits = choose_splits_fp32(n, c->sm_count, max_splits);
@@ -174,8 +177,8 @@ emtk_status run_network(emtk_ctx *c, const void *patches, int32_t n, float *cons
 }
 
 // Fills a table from requests [r0, r1); returns total hits and image bytes.
-void build_table(const emtk_ctx *c, const emtk_request *reqs, int r0, int r1, emtk_patch_format fmt, ReqTable &t,
-                 int64_t &hits, size_t &img_bytes) {
+void build_table(const emtk_ctx *c, const emtk_request *reqs, int r0, int r1, emtk_patch_format fmt, int halo,
+                 ReqTable &t, int64_t &hits, size_t &img_bytes) {
     std::memset(&t, 0, sizeof(t));
     t.n = r1 - r0;
     hits = 0;
@@ -191,13 +194,15 @@ void build_table(const emtk_ctx *c, const emtk_request *reqs, int r0, int r1, em
         d.nticks = q.nticks;
         d.nhits = q.nhits;
         d.nint = q.nticks / kDs;
-        d.pitch = (d.nint + 7) / 8 * 8;
+        d.pitch = (d.nint + 2 * halo + 7) / 8 * 8;
+        d.halo = halo;
         d.hit_begin = hits;
         d.d_off = elems;
         hits += q.nhits;
-        elems += (int64_t)d.nwires * d.pitch;
+        elems += (int64_t)(d.nwires + 2 * halo) * d.pitch;
     }
-    img_bytes = (size_t)elems * patch_elem_bytes(fmt);
+    // 64 bytes of slack: window rows are read with aligned 16-byte loads
+    img_bytes = (size_t)elems * patch_elem_bytes(fmt) + 64;
     (void)c;
 }
 
@@ -210,7 +215,8 @@ emtk_status run_requests(emtk_ctx *c, const emtk_request *reqs, int32_t nreq, cu
         const int r1 = std::min<int>(nreq, r0 + kMaxReqPerLaunch);
         int64_t hits;
         size_t img_bytes;
-        build_table(c, reqs, r0, r1, fmt, *t, hits, img_bytes);
+        const bool tc = tensor_precision(c->opt.precision);
+        build_table(c, reqs, r0, r1, fmt, tc ? kHalo : 0, *t, hits, img_bytes);
         if (hits == 0) continue;
         // planes of requests without hits need no interval image
         for (int i = 0; i < t->n; ++i)
@@ -230,13 +236,17 @@ emtk_status run_requests(emtk_ctx *c, const emtk_request *reqs, int32_t nreq, cu
             const int32_t cnt = (int32_t)std::min<int64_t>(c->max_hits, hits - g0);
             {
                 Prof prof(c, EMTK_KERNEL_GATHER, s);
-                e = launch_gather(*t, c->ws.dimg, fmt, g0, cnt, c->ws.patches, c->ws.dest, out_stride(c), s);
+                if (tc)  // the tensor-core kernel reads the windows straight from the images
+                    e = launch_hit_desc(*t, g0, cnt, c->ws.hdesc, c->ws.dest, out_stride(c), s);
+                else
+                    e = launch_gather(*t, c->ws.dimg, fmt, g0, cnt, c->ws.patches, c->ws.dest, out_stride(c), s);
             }
             if (e != cudaSuccess) {
                 st = cuda_status(e);
                 break;
             }
-            st = run_network(c, c->ws.patches, cnt, c->ws.dest, s);
+            st = tc ? run_network(c, c->ws.dimg, c->ws.hdesc, cnt, c->ws.dest, s)
+                    : run_network(c, c->ws.patches, nullptr, cnt, c->ws.dest, s);
         }
         c->stats.hits += hits;
     }
@@ -326,6 +336,8 @@ emtk_status emtk_create(const emtk_weights *w, const emtk_options *opt, int devi
     }
     if (e == cudaSuccess) e = dmalloc(&c->ws.patches, (size_t)o.max_hits * kPatchElems * patch_elem_bytes(fmt));
     if (e == cudaSuccess) e = dmalloc(&c->ws.dest, (size_t)o.max_hits * sizeof(float *));
+    if (e == cudaSuccess && tensor_precision(o.precision))
+        e = dmalloc(&c->ws.hdesc, (size_t)o.max_hits * sizeof(HitDesc));
     if (e == cudaSuccess) {
         c->ws.partial_elems = (size_t)std::max<int64_t>(kPartialCap, (int64_t)n_pad_of(o.max_hits) * kN1);
         e = dmalloc(&c->ws.partials, c->ws.partial_elems * sizeof(float));
@@ -389,7 +401,7 @@ emtk_status emtk_extract_patches(emtk_ctx *c, const float *d_adc, int32_t nwires
     if (!t) return EMTK_ERR_OOM;
     int64_t hits;
     size_t img_bytes;
-    build_table(c, &q, 0, 1, fmt, *t, hits, img_bytes);
+    build_table(c, &q, 0, 1, fmt, 0, *t, hits, img_bytes);
     st = ensure_dimg(c, img_bytes, s);
     if (st == EMTK_OK) {
         Prof prof(c, EMTK_KERNEL_INTERVALS, s);
@@ -428,7 +440,7 @@ emtk_status emtk_infer_patches(emtk_ctx *c, const float *d_patches, int32_t n, f
             Prof prof(c, EMTK_KERNEL_CONVERT, s);
             st = cuda_status(launch_fill_dest(d_scores + h0 * out_stride(c), out_stride(c), c->ws.dest, cnt, s));
         }
-        if (st == EMTK_OK) st = run_network(c, net_in, cnt, c->ws.dest, s);
+        if (st == EMTK_OK) st = run_network(c, net_in, nullptr, cnt, c->ws.dest, s);
     }
     c->stats.calls++;
     c->stats.hits += (uint64_t)n;

@@ -247,10 +247,70 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
            ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
 }
 
+// One 48-wide row of a hit's window, 16-bit pixels packed two per word:
+// element e0 of src and the 47 after it.  Seven aligned 16-byte loads cover
+// it; the words are then moved down by e0 % 8 elements with selects and a
+// funnel shift (no dynamic register indexing).  src must have 16 bytes of
+// readable memory past the last window element.
+__device__ __forceinline__ void load_window_row(const uint16_t *__restrict__ src, int64_t e0, uint32_t (&out)[24]) {
+    const int m = (int)(e0 & 7);
+    const uint4 *p = reinterpret_cast<const uint4 *>(src + (e0 - m));
+    uint32_t w[28];
+#pragma unroll
+    for (int c = 0; c < 6; ++c) {
+        const uint4 v = __ldg(p + c);
+        w[4 * c] = v.x;
+        w[4 * c + 1] = v.y;
+        w[4 * c + 2] = v.z;
+        w[4 * c + 3] = v.w;
+    }
+    if (m == 0) {
+#pragma unroll
+        for (int j = 0; j < 24; ++j) out[j] = w[j];
+        return;
+    }
+    const uint4 v = __ldg(p + 6);
+    w[24] = v.x;
+    w[25] = v.y;
+    w[26] = v.z;
+    w[27] = v.w;
+    const int s = m >> 1;
+    uint32_t a[26];
+#pragma unroll
+    for (int j = 0; j < 26; ++j) a[j] = (s & 2) ? w[j + 2] : w[j];
+    uint32_t b[25];
+#pragma unroll
+    for (int j = 0; j < 25; ++j) b[j] = (s & 1) ? a[j + 1] : a[j];
+    if (m & 1) {
+#pragma unroll
+        for (int j = 0; j < 24; ++j) out[j] = __funnelshift_r(b[j], b[j + 1], 16);
+    } else {
+#pragma unroll
+        for (int j = 0; j < 24; ++j) out[j] = b[j];
+    }
+}
+
+// The same row for a hit whose window leaves the haloed image (a hit outside
+// its plane): every pixel checked against the plane, zero outside.
+__device__ __forceinline__ void load_window_row_checked(const uint16_t *__restrict__ src, const HitDesc &hd, int r,
+                                                     uint32_t (&out)[24]) {
+    const int w = hd.wc - kHalf + r;
+    const bool wok = w >= 0 && w < hd.nwires;
+    const uint16_t *rowp = src + hd.d_off + (int64_t)(wok ? w + kHalo : 0) * hd.pitch + kHalo;
+#pragma unroll
+    for (int j = 0; j < 24; ++j) {
+        const int64_t b0 = (int64_t)hd.bc - kHalf + 2 * j;
+        const uint32_t lo = (wok && b0 >= 0 && b0 < hd.nint) ? rowp[b0] : 0u;
+        const uint32_t hi = (wok && b0 + 1 >= 0 && b0 + 1 < hd.nint) ? rowp[b0 + 1] : 0u;
+        out[j] = lo | (hi << 16);
+    }
+}
+
 // ------------------------------------------------------------------ kernel
 template <bool FP16>
 __global__ void __launch_bounds__(kThreadsTC, 1)
-    cnn_tc_kernel(const __grid_constant__ CUtensorMap tmap_w1, const uint16_t *__restrict__ patches, int n,
+    cnn_tc_kernel(const __grid_constant__ CUtensorMap tmap_w1, const uint16_t *__restrict__ src,
+                  const HitDesc *__restrict__ desc, int n,
                   const uint16_t *__restrict__ convB_g, float *__restrict__ partials, int n_pad, long long units,
                   int *status, long long timeout_ns, int debug_stall) {
     extern __shared__ uint8_t smem_raw[];
@@ -461,20 +521,30 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         const int64_t k_base = (int64_t)tile * kW1Steps - u0;        // running quad index = k_base + quad
         const int64_t hit = (int64_t)tile * 128 + row;
         const bool valid = hit < n;
-        const uint4 *prow = reinterpret_cast<const uint4 *>(patches) + (valid ? hit : 0) * (kPatchElems / 8);
+        // the hit's window: a patch of the patch buffer, or a window of its plane's image
+        HitDesc hd;
+        if (desc == nullptr) {
+            hd.origin = valid ? hit * kPatchElems : 0;
+            hd.pitch = kPatch;
+            hd.inside = 1;
+        } else if (valid) {
+            hd = desc[hit];
+        } else {
+            hd.inside = 1;
+        }
         const int y_first = j0 * kPosPerW1 / kQ;
         const int y_last = (j1 * kPosPerW1 - 1) / kQ;
         for (int y = y_first; ok && y <= y_last; ++y) {
-            uint32_t R[kK][24];  // patch rows y..y+4 of this hit, 2 pixels per word
+            uint32_t R[kK][24];  // window rows y..y+4 of this hit, 2 pixels per word
 #pragma unroll
             for (int i = 0; i < kK; ++i) {
+                if (!valid) {
 #pragma unroll
-                for (int u = 0; u < 6; ++u) {
-                    const uint4 v = valid ? __ldg(prow + (y + i) * 6 + u) : make_uint4(0u, 0u, 0u, 0u);
-                    R[i][4 * u + 0] = v.x;
-                    R[i][4 * u + 1] = v.y;
-                    R[i][4 * u + 2] = v.z;
-                    R[i][4 * u + 3] = v.w;
+                    for (int j = 0; j < 24; ++j) R[i][j] = 0u;
+                } else if (hd.inside) {
+                    load_window_row(src, hd.origin + (int64_t)(y + i) * hd.pitch, R[i]);
+                } else {
+                    load_window_row_checked(src, hd, y + i, R[i]);
                 }
             }
 #pragma unroll
@@ -689,19 +759,19 @@ int streamk_partial_rows(int32_t n, int G) {
     return rows;
 }
 
-cudaError_t launch_cnn_tc(const DeviceWeights &w, const void *patches, bool fp16, int32_t n, int G,
-                          float *partials, int n_pad, int *status, int64_t timeout_ns, int debug_stall,
+cudaError_t launch_cnn_tc(const DeviceWeights &w, const void *src, const HitDesc *desc, bool fp16, int32_t n,
+                          int G, float *partials, int n_pad, int *status, int64_t timeout_ns, int debug_stall,
                           cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
     const CUtensorMap &map = *static_cast<const CUtensorMap *>(w.w1_tmap);
     const long long units = (long long)((n + 127) / 128) * kW1Steps;
     dim3 grid(G);
     if (fp16)
-        cnn_tc_kernel<true><<<grid, kThreadsTC, kSmemBytesTC, s>>>(map, static_cast<const uint16_t *>(patches), n,
+        cnn_tc_kernel<true><<<grid, kThreadsTC, kSmemBytesTC, s>>>(map, static_cast<const uint16_t *>(src), desc, n,
                                                                    w.convB, partials, n_pad, units, status,
                                                                    (long long)timeout_ns, debug_stall);
     else
-        cnn_tc_kernel<false><<<grid, kThreadsTC, kSmemBytesTC, s>>>(map, static_cast<const uint16_t *>(patches), n,
+        cnn_tc_kernel<false><<<grid, kThreadsTC, kSmemBytesTC, s>>>(map, static_cast<const uint16_t *>(src), desc, n,
                                                                     w.convB, partials, n_pad, units, status,
                                                                     (long long)timeout_ns, debug_stall);
     return cudaGetLastError();

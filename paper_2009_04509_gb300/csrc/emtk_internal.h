@@ -52,9 +52,24 @@ struct ReqDesc {
     int32_t nticks;
     int32_t nhits;
     int32_t nint;         // complete time intervals: nticks / 6
-    int32_t pitch;        // row pitch of the interval image: nint rounded up to 8
-    int32_t pad;
+    int32_t pitch;        // row pitch of the interval image (a multiple of 8 elements)
+    int32_t halo;         // zero border of the image: element (w, b) is at
+                          // d_off + (w + halo) * pitch + (b + halo); rows nwires + 2 halo
 };
+
+// Where the tensor-core kernel finds a hit's 48 x 48 window: element (r, c)
+// is src[origin + r * pitch + c] when `inside` (the whole window lies in the
+// haloed image); otherwise it is the image pixel (wc - 24 + r, bc - 24 + c)
+// of the plane at d_off, zero outside [0, nwires) x [0, nint).
+struct HitDesc {
+    int64_t origin;
+    int64_t d_off;
+    int32_t pitch;
+    int32_t inside;
+    int32_t wc, bc;
+    int32_t nwires, nint;
+};
+constexpr int kHalo = kHalf;    // image border for the tensor-core path
 
 struct ReqTable {
     int32_t n;
@@ -67,6 +82,7 @@ struct Workspace {
     void *dimg = nullptr;        // interval images of the planes of one launch
     size_t dimg_bytes = 0;
     void *patches = nullptr;     // [max_hits][48][48] in the precision's patch format
+    HitDesc *hdesc = nullptr;    // [max_hits] window descriptors (tensor-core path)
     float **dest = nullptr;      // [max_hits] output row of each hit
     float *partials = nullptr;   // [max_splits][max_hits_pad][128]
     size_t partial_elems = 0;
@@ -121,6 +137,10 @@ cudaError_t launch_gather(const ReqTable &t, const void *dimg, emtk_patch_format
 // Patch cut straight from the planes into caller memory (emtk_extract_patches).
 cudaError_t launch_convert_patches(const float *src, void *dst, emtk_patch_format fmt, int64_t n,
                                    cudaStream_t s);
+// Window descriptors of hits [g0, g0+count) (images with halo kHalo), and
+// the output row of each hit in dest.
+cudaError_t launch_hit_desc(const ReqTable &t, int64_t g0, int32_t count, HitDesc *desc, float **dest,
+                            int out_stride, cudaStream_t s);
 cudaError_t launch_fill_dest(float *scores, int out_stride, float **dest, int32_t n, cudaStream_t s);
 
 // Network: dense-1 partial sums [splits][n_pad][128] from patches.
@@ -128,8 +148,10 @@ cudaError_t launch_cnn_fp32(const DeviceWeights &w, const float *patches, int32_
                             float *partials, int n_pad, cudaStream_t s);
 // Stream-K over G CTAs (one per SM); partials [rows][n_pad][128] with rows
 // = streamk_partial_rows(n, G).
-cudaError_t launch_cnn_tc(const DeviceWeights &w, const void *patches, bool fp16, int32_t n, int G,
-                          float *partials, int n_pad, int *status, int64_t timeout_ns, int debug_stall,
+// src: 16-bit patches [n][48][48] (desc == nullptr) or the haloed interval
+// images of the hits' planes, located through desc.
+cudaError_t launch_cnn_tc(const DeviceWeights &w, const void *src, const HitDesc *desc, bool fp16, int32_t n,
+                          int G, float *partials, int n_pad, int *status, int64_t timeout_ns, int debug_stall,
                           cudaStream_t s);
 int streamk_partial_rows(int32_t n, int G);
 // Sum of partials + bias + ReLU, dense-2, heads; scores to dest[h].  Partial

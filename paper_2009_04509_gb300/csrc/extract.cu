@@ -57,32 +57,38 @@ __device__ __forceinline__ void store2(void *base, int64_t idx, float v0, float 
     }
 }
 
-// One thread = two consecutive intervals of one wire (12 ticks = 48 bytes,
-// 16-byte aligned because ld % 4 == 0 and the plane is 16-byte aligned).
-// grid.y = request; image rows have an even pitch and start at an even
-// element offset, so the pair store is aligned too.
+// One thread = two consecutive image columns of one image row; inside the
+// plane that is two intervals of one wire (12 ticks = 48 bytes, 16-byte
+// aligned because ld % 4 == 0, the plane is 16-byte aligned and the halo is
+// even), outside it (the zero halo, the pitch padding) zeros.  grid.y =
+// request; the pitch and the image offset are even, so the pair store is
+// aligned too.
 template <int FMT>
 __global__ void __launch_bounds__(256) interval_image_kernel(const __grid_constant__ ReqTable t, void *img) {
     const ReqDesc &r = t.r[blockIdx.y];
-    const int npairs = (r.nint + 1) >> 1;
-    const int64_t work = (int64_t)r.nwires * npairs;
+    if (r.nwires == 0) return;
+    const int npairs = r.pitch >> 1;
+    const int rows = r.nwires + 2 * r.halo;
+    const int64_t work = (int64_t)rows * npairs;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < work;
          i += (int64_t)gridDim.x * blockDim.x) {
-        const int w = (int)(i / npairs);
-        const int bp = (int)(i - (int64_t)w * npairs);
-        const int b = 2 * bp;
-        const float *src = r.adc + (int64_t)w * r.ld + 6 * b;
-        const bool two = (b + 1) < r.nint;
-        const float4 x0 = __ldcs(reinterpret_cast<const float4 *>(src));
-        const float2 x1 = __ldcs(reinterpret_cast<const float2 *>(src + 4));
-        const float v0 = interval_sum(x0.x, x0.y, x0.z, x0.w, x1.x, x1.y);
-        float v1 = 0.0f;
-        if (two) {
-            const float2 x2 = __ldcs(reinterpret_cast<const float2 *>(src + 6));
-            const float4 x3 = __ldcs(reinterpret_cast<const float4 *>(src + 8));
-            v1 = interval_sum(x2.x, x2.y, x3.x, x3.y, x3.z, x3.w);
+        const int wr = (int)(i / npairs);
+        const int cb = 2 * (int)(i - (int64_t)wr * npairs);
+        const int w = wr - r.halo;
+        const int b = cb - r.halo;
+        float v0 = 0.0f, v1 = 0.0f;
+        if (w >= 0 && w < r.nwires && b >= 0 && b < r.nint) {
+            const float *src = r.adc + (int64_t)w * r.ld + 6 * b;
+            const float4 x0 = __ldcs(reinterpret_cast<const float4 *>(src));
+            const float2 x1 = __ldcs(reinterpret_cast<const float2 *>(src + 4));
+            v0 = interval_sum(x0.x, x0.y, x0.z, x0.w, x1.x, x1.y);
+            if (b + 1 < r.nint) {
+                const float2 x2 = __ldcs(reinterpret_cast<const float2 *>(src + 6));
+                const float4 x3 = __ldcs(reinterpret_cast<const float4 *>(src + 8));
+                v1 = interval_sum(x2.x, x2.y, x3.x, x3.y, x3.z, x3.w);
+            }
         }
-        store2<FMT>(img, r.d_off + (int64_t)w * r.pitch + b, v0, v1, two);
+        store2<FMT>(img, r.d_off + (int64_t)wr * r.pitch + cb, v0, v1, true);
     }
 }
 
@@ -150,7 +156,7 @@ __global__ void __launch_bounds__(288) gather_kernel(const __grid_constant__ Req
 #pragma unroll
         for (int e = 0; e < V; ++e) {
             const int64_t b = bc - kHalf + c0 + e;
-            v.e[e] = (wire_ok && b >= 0 && b < r.nint) ? src[w * r.pitch + b] : T(0);
+            v.e[e] = (wire_ok && b >= 0 && b < r.nint) ? src[(w + r.halo) * r.pitch + b + r.halo] : T(0);
         }
         *reinterpret_cast<uint4 *>(out + row * kPatch + c0) = v.u;
     }
@@ -167,6 +173,30 @@ __global__ void convert_kernel(const float *src, void *dst, int64_t n) {
     }
 }
 
+__global__ void hit_desc_kernel(const __grid_constant__ ReqTable t, int64_t g0, int32_t count, HitDesc *desc,
+                                float **dest, int out_stride) {
+    const int64_t local = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (local >= count) return;
+    const int64_t g = g0 + local;
+    const ReqDesc &r = t.r[find_request(t, g)];
+    const int64_t hloc = g - r.hit_begin;
+    const emtk_hit hit = r.hits[hloc];
+    const int64_t bc = floor_div6(hit.tick);
+    HitDesc d;
+    d.wc = hit.wire;
+    d.bc = (int32_t)bc;  // |tick| < 2^31, so the interval fits
+    d.nwires = r.nwires;
+    d.nint = r.nint;
+    d.pitch = r.pitch;
+    d.d_off = r.d_off;
+    // the window [wc-24, wc+24) x [bc-24, bc+24) lies in the haloed image iff
+    // the hit itself lies in the plane (the halo is 24 wide)
+    d.inside = (hit.wire >= 0 && hit.wire < r.nwires && bc >= 0 && bc < r.nint) ? 1 : 0;
+    d.origin = d.inside ? r.d_off + (int64_t)(hit.wire - kHalf + r.halo) * r.pitch + (bc - kHalf + r.halo) : 0;
+    desc[local] = d;
+    if (dest != nullptr) dest[local] = r.scores + hloc * out_stride;
+}
+
 __global__ void fill_dest_kernel(float *scores, int stride, float **dest, int32_t n) {
     const int i = blockIdx.x * blockDim.x + threadIdx.x;
     if (i < n) dest[i] = scores + (int64_t)i * stride;
@@ -177,7 +207,7 @@ __global__ void fill_dest_kernel(float *scores, int stride, float **dest, int32_
 cudaError_t launch_interval_images(const ReqTable &t, void *dimg, emtk_patch_format fmt, cudaStream_t s) {
     int64_t most = 0;
     for (int i = 0; i < t.n; ++i) {
-        const int64_t w = (int64_t)t.r[i].nwires * ((t.r[i].nint + 1) / 2);
+        const int64_t w = t.r[i].nwires ? (int64_t)(t.r[i].nwires + 2 * t.r[i].halo) * (t.r[i].pitch / 2) : 0;
         most = w > most ? w : most;
     }
     if (most == 0 || t.n == 0) return cudaSuccess;
@@ -213,6 +243,13 @@ cudaError_t launch_convert_patches(const float *src, void *dst, emtk_patch_forma
         convert_kernel<EMTK_PATCH_BF16><<<(unsigned)blocks, 256, 0, s>>>(src, dst, n);
     else
         convert_kernel<EMTK_PATCH_F16><<<(unsigned)blocks, 256, 0, s>>>(src, dst, n);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_hit_desc(const ReqTable &t, int64_t g0, int32_t count, HitDesc *desc, float **dest,
+                            int out_stride, cudaStream_t s) {
+    if (count <= 0) return cudaSuccess;
+    hit_desc_kernel<<<(count + 255) / 256, 256, 0, s>>>(t, g0, count, desc, dest, out_stride);
     return cudaGetLastError();
 }
 

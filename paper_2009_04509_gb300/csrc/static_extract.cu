@@ -87,7 +87,7 @@ extern "C" emtk_status emtk_extract_patches_static(const float *d_adc, int32_t n
     d.nhits = nhits;
     d.nint = nint;
     d.pitch = pitch;
-    d.pad = 0;
+    d.halo = 0;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     if (launch_interval_images(t, img, fmt, s) != cudaSuccess) return EMTK_ERR_CUDA;
     if (launch_gather(t, img, fmt, 0, nhits, d_patches, nullptr, 0, s) != cudaSuccess) return EMTK_ERR_CUDA;
