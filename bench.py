@@ -251,7 +251,10 @@ def main():
     flop_net = (FLOP_CONV + FLOP_FC1) * hits_per_launch
     achieved = flop_net / (net_ms / 1e3) / 1e12
     union = window_union_bytes(planes)
-    patch_bytes = nhits * 48 * 48 * (4 if args.precision == "fp32" else 2)
+    if args.precision == "fp32":  # the fp32 path writes every patch
+        patch_bytes = nhits * 48 * 48 * 4
+    else:  # the 16-bit paths write the interval image; the network reads the windows from it
+        patch_bytes = sum(p.nwires * (p.nticks // 6) for p in planes) * 2
     cut_ms = (kms["intervals"] + kms["gather"]) / args.steps
     cut_gbs = (union + patch_bytes) / (cut_ms / 1e3) / 1e9
 
@@ -289,6 +292,9 @@ def main():
                      "launch_ms": net_ms, "traffic": None},
         "extraction": {"bound": "hbm", "achieved": cut_gbs, "peak": peaks["hbm"], "unit": "GB/s",
                        "frac": cut_gbs / peaks["hbm"], "algorithmic_bytes": union + patch_bytes,
+                       "bytes_read": union, "bytes_written": patch_bytes,
+                       "kernels": "interval_image_kernel + " + ("gather_kernel" if args.precision == "fp32"
+                                                               else "hit_desc_kernel"),
                        "ms_per_step": cut_ms},
         "kernel_ms_per_step": {k: v / args.steps for k, v in kms.items()},
         "whole_step_frac_of_bf16_peak": value * FLOP_PER_HIT / 1e12 / peaks["bf16"] / world,
