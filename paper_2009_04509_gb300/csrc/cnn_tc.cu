@@ -36,8 +36,20 @@
 namespace emtk {
 namespace {
 
-constexpr int kThreadsTC = 352;  // warp 0 TMA, warp 1 conv MMA, 2-5 builder, 6-9 epilogue, 10 dense-1 MMA
-constexpr int kFc1Warp = 10;
+// Warp roles.  A warp runs on the SM sub-partition (scheduler) warp mod 4,
+// and an epilogue warp may only touch TMEM lanes 32 (warp mod 4) .. +31, so
+// the four epilogue warps sit on all four sub-partitions.  The dense-1
+// issuer, whose every idle cycle between MMAs idles the tensor pipe, shares
+// its sub-partition with one epilogue warp only; the builder warps take the
+// other slots.
+constexpr int kThreadsTC = 352;  // 11 warps
+constexpr int kTmaWarp = 0;
+constexpr int kConvWarp = 1;
+constexpr int kFc1Warp = 3;
+constexpr int kEpiWarp0 = 4;     // warps 4-7: epilogue, TMEM lane quarter warp mod 4
+__host__ __device__ constexpr int builder_index(int warp) {  // warps 2, 8, 9, 10 -> row blocks 0-3
+    return warp == 2 ? 0 : warp >= 8 ? warp - 7 : -1;
+}
 constexpr int kW1Stages = 3;     // shared-memory stages of W1 (one quad each)
 constexpr int kImBufs = 3;       // shared-memory im2col tiles (one quad each)
 constexpr int kSlots = 4;        // TMEM conv/activation slots (one pair each)
@@ -364,7 +376,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    if (warp == 1) {
+    if (warp == kConvWarp) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(base + kOffTmemSlot),
                      "r"(kTmemCols)
                      : "memory");
@@ -375,7 +387,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    if (warp == 0) {
+    if (warp == kTmaWarp) {
         // ================================================= TMA producer (W1)
         if (lane == 0) {
             int issued = 0;
@@ -409,9 +421,9 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 }
             }
         }
-    } else if (warp == 1 || warp == kFc1Warp) {
+    } else if (warp == kConvWarp || warp == kFc1Warp) {
         // ====================================================== MMA issuers
-        // Two threads issue MMAs, lane 0 of warp 1 (the convs) and lane 0 of
+        // Two threads issue MMAs, lane 0 of warp kConvWarp (the convs) and lane 0 of
         // warp kFc1Warp (dense-1); each walks its own schedule alone, so that
         // nothing but its waits stands between its groups of MMAs (the tensor
         // pipe's queue is shallow: an issuing thread runs at the pace of
@@ -424,7 +436,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         // all earlier MMAs of its thread.
         if (lane == 0) {
             bool ok = true;
-            if (warp == 1) {
+            if (warp == kConvWarp) {
                 constexpr uint32_t idesc_conv = make_idesc(128, kPairN, FP16);
                 const uint64_t convb_desc = sw128_desc(sConvB);
                 if (debug_stall) ok = wait_bounded(bar(kBarStall), 0u, guard);  // nothing arrives here
@@ -500,14 +512,14 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
             }
         }
         __syncwarp();
-    } else if (warp < 6) {
+    } else if (builder_index(warp) >= 0) {
         // ================================================ im2col builder
         // Row r of an im2col tile (hit r) is 128 bytes: pair (x, x+1) in
         // chunks 0-3, pair (x+2, x+3) in chunks 4-7; 16-byte chunk c sits at
         // chunk c ^ (r & 7) (128-byte swizzle).  Tap t = 6i + j of a pair at x
         // is patch pixel (y + i, x + j); taps 30 and 31 are 1.0.  Because x is
         // even, taps (2k, 2k+1) are one aligned pixel pair of the patch row.
-        const int q4 = warp & 3;
+        const int q4 = builder_index(warp);
         const int row = 32 * q4 + lane;
         const uint32_t one = FP16 ? 0x3C00u : 0x3F80u;
         const uint32_t ones = one | (one << 16);
@@ -581,7 +593,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
             }
         }
         }
-    } else if (warp < kFc1Warp) {
+    } else {
         // ================================== conv epilogue + dense-1 store
         const int q4 = warp & 3;
         const int row = 32 * q4 + lane;
@@ -654,7 +666,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
 
     tc_fence_before();
     __syncthreads();
-    if (warp == 1) {
+    if (warp == kConvWarp) {
         __syncwarp();
         tc_fence_after();
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
