@@ -546,19 +546,29 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         }
         const int y_first = j0 * kPosPerW1 / kQ;
         const int y_last = (j1 * kPosPerW1 - 1) / kQ;
-        for (int y = y_first; ok && y <= y_last; ++y) {
-            uint32_t R[kK][24];  // window rows y..y+4 of this hit, 2 pixels per word
+        // window row r of this hit, 2 pixels per word
+        auto load_row = [&](int r, uint32_t(&out)[24]) {
+            if (!valid) {
 #pragma unroll
-            for (int i = 0; i < kK; ++i) {
-                if (!valid) {
-#pragma unroll
-                    for (int j = 0; j < 24; ++j) R[i][j] = 0u;
-                } else if (hd.inside) {
-                    load_window_row(src, hd.origin + (int64_t)(y + i) * hd.pitch, R[i]);
-                } else {
-                    load_window_row_checked(src, hd, y + i, R[i]);
-                }
+                for (int j = 0; j < 24; ++j) out[j] = 0u;
+            } else if (hd.inside) {
+                load_window_row(src, hd.origin + (int64_t)r * hd.pitch, out);
+            } else {
+                load_window_row_checked(src, hd, r, out);
             }
+        };
+        // rows y..y+4, slid down one row per y: each window row is loaded once
+        uint32_t R[kK][24];
+#pragma unroll
+        for (int i = 0; i < kK - 1; ++i) load_row(y_first + i, R[i]);
+        for (int y = y_first; ok && y <= y_last; ++y) {
+            if (y > y_first) {
+#pragma unroll
+                for (int i = 0; i < kK - 1; ++i)
+#pragma unroll
+                    for (int j = 0; j < 24; ++j) R[i][j] = R[i + 1][j];
+            }
+            load_row(y + kK - 1, R[kK - 1]);
 #pragma unroll
             for (int xq = 0; xq < kQ / kPosPerW1; ++xq) {
                 const int quad = (y * kQ) / kPosPerW1 + xq;
