@@ -477,7 +477,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                     const int s0 = (2 * q) % kSlots, s1 = (2 * q + 1) % kSlots;
                     const uint32_t par = (uint32_t)((2 * q) / kSlots) & 1u;  // same use for both slots
                     if (!wait_bounded(bar(kBarW1Full + wj), (uint32_t)(q / kW1Stages) & 1u, guard) ||
-                        !wait_bounded(bar(kBarAct + s0), par, guard) || !wait_bounded(bar(kBarAct + s1), par, guard)) {
+                        !wait_bounded(bar(kBarAct + s0), par, guard)) {
                         ok = false;
                         break;
                     }
@@ -491,11 +491,20 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                     const uint64_t wdesc = sw128_desc(sW1 + wj * kW1StageBytes);
 #pragma unroll
                     for (int step = 0; step < 12; ++step) {  // 16-wide K steps of the quad's 192
+                        // the second pair's activations are waited for only when its half begins
+                        if (step == 6) {
+                            if (!wait_bounded(bar(kBarAct + s1), par, guard)) {
+                                ok = false;
+                                break;
+                            }
+                            tc_fence_after();
+                        }
                         const uint32_t a = tmem + kSlotCol0 + (uint32_t)(step < 6 ? s0 : s1) * kSlotCols + 8u * (step % 6);
                         const uint64_t bd = wdesc + (uint64_t)(((step >> 2) * kW1BoxBytes + (step & 3) * 32) >> 4);
                         mma_ts(tmem + kAccCol, a, bd, idesc_fc1, (first && step == 0) ? 0u : 1u);
                         if (step == 5) mma_commit(bar(kBarFree + s0));
                     }
+                    if (!ok) break;
                     mma_commit(bar(kBarFree + s1));
                     mma_commit(bar(kBarW1Empty + wj));
                     if (last) {
