@@ -33,6 +33,21 @@ FLOP_TAIL = 2 * (128 * 32 + 32 * 4)         # 8,448
 FLOP_PER_HIT = FLOP_CONV + FLOP_FC1 + FLOP_TAIL  # 28,444,416
 METRIC = "hit patches/sec on 1 GB300 (extract+CNN); % bf16 tensor peak; gather HBM GB/s"
 
+# DRAM bytes (read + write) of one cnn_tc_kernel launch on the full event, bf16, from
+# one ncu capture of this benchmark (profiles/launch_list_full_event_bf16.md), valid
+# for the kernel source it was taken on: reported as null once that source changes.
+TC_TRAFFIC_BYTES = 50_807_040 + 6_299_904
+TC_TRAFFIC_SOURCE_SHA256 = "16fb956eebfa43b0"
+
+
+def tc_traffic(precision: str, workload: str):
+    import hashlib
+    src = os.path.join(ROOT, "paper_2009_04509_gb300", "csrc", "cnn_tc.cu")
+    if precision != "bf16" or workload != "full_event" or not os.path.exists(src):
+        return None
+    h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    return TC_TRAFFIC_BYTES if h == TC_TRAFFIC_SOURCE_SHA256 else None
+
 
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
@@ -289,7 +304,8 @@ def main():
                      "frac": achieved / peaks["bf16_sus"],
                      "peak_source": f"{peaks['source']} bf16 sustained", "frac_of_burst": achieved / peaks["bf16"],
                      "flop_per_hit": FLOP_CONV + FLOP_FC1, "hits_per_launch": hits_per_launch,
-                     "launch_ms": net_ms, "traffic": None},
+                     "launch_ms": net_ms, "traffic": tc_traffic(args.precision, args.workload),
+                     "traffic_unit": "bytes per launch (ncu dram__bytes_read.sum + dram__bytes_write.sum)"},
         "extraction": {"bound": "hbm", "achieved": cut_gbs, "peak": peaks["hbm"], "unit": "GB/s",
                        "frac": cut_gbs / peaks["hbm"], "algorithmic_bytes": union + patch_bytes,
                        "bytes_read": union, "bytes_written": patch_bytes,
