@@ -212,6 +212,54 @@ EMTK_API emtk_status emtk_get_stats(emtk_ctx *ctx, emtk_stats *out);
 /* Static English text for a status code. */
 EMTK_API const char *emtk_status_string(emtk_status s);
 
+/* ------------------------------------------------------------------------
+ * Request batcher: many clients, one GPU.
+ *
+ * In the paper's setup (Sec. 2.3, 3.2) many CPU processes send inference
+ * requests to a server whose dynamic batching merges them into larger
+ * batches.  The batcher is that merging step inside one process: client
+ * threads submit requests (a plane and its hit list, emtk_request) and wait
+ * for their scores; a dispatcher thread forms batches of whole requests and
+ * runs each with emtk_infer_batch on one of the batcher's own CUDA streams,
+ * each stream with its own workspace (the weights of `ctx` are shared).
+ *   - A batch is launched when its requests hold max_hits hits, or when its
+ *     oldest request has waited max_delay_us, whichever comes first.  A
+ *     request larger than max_hits goes alone.  Requests leave in
+ *     submission order.
+ *   - The request's buffers (d_adc, d_hits, d_scores) must stay valid and
+ *     unchanged until emtk_batcher_wait() has returned for its ticket; they
+ *     are read and written on the batcher's streams, not the caller's.
+ *   - ctx must outlive the batcher and must not be used from other threads
+ *     while the batcher exists; its precision and options apply.
+ * -------------------------------------------------------------------- */
+typedef struct emtk_batcher emtk_batcher;
+
+/* nstreams in [1, 16]; max_hits > 0; max_delay_us >= 0.  Creates the
+ * streams and workspaces (device allocations) and starts the dispatcher and
+ * completion threads. */
+EMTK_API emtk_status emtk_batcher_create(emtk_ctx *ctx, int32_t nstreams, int32_t max_hits, int64_t max_delay_us,
+                                         emtk_batcher **out);
+
+/* Thread-safe, non-blocking: queues one request and returns its ticket (> 0).
+ * The request is checked as emtk_infer_batch checks it; an invalid one
+ * returns that status and is not queued. */
+EMTK_API emtk_status emtk_batcher_submit(emtk_batcher *b, const emtk_request *req, uint64_t *ticket);
+
+/* Thread-safe: blocks until the ticket's scores are complete in device
+ * memory, then returns the status of its batch (EMTK_ERR_TIMEOUT if a
+ * device-side wait of that batch gave up).  Returns EMTK_ERR_TIMEOUT after
+ * timeout_ms (< 0: no limit) without consuming the ticket, and EMTK_ERR_ARG
+ * for a ticket that was never issued or was already waited for. */
+EMTK_API emtk_status emtk_batcher_wait(emtk_batcher *b, uint64_t ticket, int64_t timeout_ms);
+
+/* Counters since creation: batches launched, requests and hits in them. */
+EMTK_API emtk_status emtk_batcher_stats(emtk_batcher *b, int64_t *batches, int64_t *requests, int64_t *hits);
+
+/* Launches what is still queued, waits for every batch, stops the threads
+ * and frees the batcher's streams and workspaces.  NULL is allowed.  Tickets
+ * not yet waited for are dropped. */
+EMTK_API emtk_status emtk_batcher_destroy(emtk_batcher *b);
+
 #ifdef __cplusplus
 }
 #endif

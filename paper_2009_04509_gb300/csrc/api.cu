@@ -60,12 +60,16 @@ void free_ctx(emtk_ctx *c) {
     if (!c) return;
     drain_events(c);
     DeviceWeights &w = c->w;
-    for (void *p : {(void *)w.conv_w, (void *)w.conv_b, (void *)w.fc1_w, (void *)w.fc1_b, (void *)w.fc2_w,
-                    (void *)w.fc2_b, (void *)w.cls_w, (void *)w.cls_b, (void *)w.mic_w, (void *)w.mic_b,
-                    (void *)w.w1_tiles, (void *)w.convB, c->ws.dimg, c->ws.patches, (void *)c->ws.dest,
-                    (void *)c->ws.partials, (void *)c->ws.status, (void *)c->ws.hdesc})
+    if (c->owns_weights) {
+        for (void *p : {(void *)w.conv_w, (void *)w.conv_b, (void *)w.fc1_w, (void *)w.fc1_b, (void *)w.fc2_w,
+                        (void *)w.fc2_b, (void *)w.cls_w, (void *)w.cls_b, (void *)w.mic_w, (void *)w.mic_b,
+                        (void *)w.w1_tiles, (void *)w.convB})
+            if (p) cudaFree(p);
+        delete static_cast<CUtensorMap *>(w.w1_tmap);
+    }
+    for (void *p : {c->ws.dimg, c->ws.patches, (void *)c->ws.dest, (void *)c->ws.partials, (void *)c->ws.status,
+                    (void *)c->ws.hdesc})
         if (p) cudaFree(p);
-    delete static_cast<CUtensorMap *>(w.w1_tmap);
     delete c;
 }
 
@@ -254,7 +258,70 @@ emtk_status run_requests(emtk_ctx *c, const emtk_request *reqs, int32_t nreq, cu
     return st;
 }
 
+// Workspace of a context, sized by its max_hits.  The patch buffer is only
+// needed by the fp32 path and emtk_infer_patches (`patches`).
+cudaError_t alloc_workspace(emtk_ctx *c, bool patches) {
+    const emtk_options &o = c->opt;
+    const emtk_patch_format fmt = patch_format(o.precision);
+    cudaError_t e = cudaSuccess;
+    if (patches || !tensor_precision(o.precision))
+        e = dmalloc(&c->ws.patches, (size_t)o.max_hits * kPatchElems * patch_elem_bytes(fmt));
+    if (e == cudaSuccess) e = dmalloc(&c->ws.dest, (size_t)o.max_hits * sizeof(float *));
+    if (e == cudaSuccess && tensor_precision(o.precision))
+        e = dmalloc(&c->ws.hdesc, (size_t)o.max_hits * sizeof(HitDesc));
+    if (e == cudaSuccess) {
+        c->ws.partial_elems = (size_t)std::max<int64_t>(kPartialCap, (int64_t)n_pad_of(o.max_hits) * kN1);
+        e = dmalloc(&c->ws.partials, c->ws.partial_elems * sizeof(float));
+    }
+    if (e == cudaSuccess) e = dmalloc(&c->ws.status, sizeof(int));
+    if (e == cudaSuccess) e = cudaMemset(c->ws.status, 0, sizeof(int));
+    return e;
+}
+
 }  // namespace
+
+namespace emtk {
+
+emtk_status validate_request(const emtk_request &q) {
+    emtk_status st = check_plane(q.d_adc, q.nwires, q.nticks, q.ld, q.d_hits, q.nhits);
+    if (st != EMTK_OK) return st;
+    if (q.nhits > 0 && q.d_scores == nullptr) return EMTK_ERR_ARG;
+    if ((reinterpret_cast<uintptr_t>(q.d_scores) & 3u) != 0) return EMTK_ERR_ALIGN;
+    return EMTK_OK;
+}
+
+emtk_ctx *make_lane_ctx(const emtk_ctx *parent, emtk_status *st) {
+    emtk_ctx *c = new (std::nothrow) emtk_ctx;
+    if (!c) {
+        *st = EMTK_ERR_OOM;
+        return nullptr;
+    }
+    c->device = parent->device;
+    c->opt = parent->opt;
+    c->opt.profile = 0;
+    c->max_hits = parent->max_hits;
+    c->sm_count = parent->sm_count;
+    c->w = parent->w;
+    c->owns_weights = false;
+    DeviceGuard g(c->device);
+    cudaError_t e = g.ok ? alloc_workspace(c, false) : cudaErrorInvalidDevice;
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) {
+        free_ctx(c);
+        *st = cuda_status(e);
+        return nullptr;
+    }
+    *st = EMTK_OK;
+    return c;
+}
+
+void destroy_lane_ctx(emtk_ctx *c) {
+    if (!c) return;
+    DeviceGuard g(c->device);
+    free_ctx(c);
+}
+
+}  // namespace emtk
 
 extern "C" {
 
@@ -313,7 +380,6 @@ emtk_status emtk_create(const emtk_weights *w, const emtk_options *opt, int devi
     c->opt = o;
     c->max_hits = o.max_hits;
     c->sm_count = prop.multiProcessorCount;
-    const emtk_patch_format fmt = patch_format(o.precision);
     cudaError_t e = cudaSuccess;
     DeviceWeights &d = c->w;
     if (e == cudaSuccess) e = upload(&d.conv_w, w->conv_w, (size_t)kK * kK * kF);
@@ -334,16 +400,7 @@ emtk_status emtk_create(const emtk_weights *w, const emtk_options *opt, int devi
             if (e == cudaSuccess) e = init_fp32_kernel_attrs();
         }
     }
-    if (e == cudaSuccess) e = dmalloc(&c->ws.patches, (size_t)o.max_hits * kPatchElems * patch_elem_bytes(fmt));
-    if (e == cudaSuccess) e = dmalloc(&c->ws.dest, (size_t)o.max_hits * sizeof(float *));
-    if (e == cudaSuccess && tensor_precision(o.precision))
-        e = dmalloc(&c->ws.hdesc, (size_t)o.max_hits * sizeof(HitDesc));
-    if (e == cudaSuccess) {
-        c->ws.partial_elems = (size_t)std::max<int64_t>(kPartialCap, (int64_t)n_pad_of(o.max_hits) * kN1);
-        e = dmalloc(&c->ws.partials, c->ws.partial_elems * sizeof(float));
-    }
-    if (e == cudaSuccess) e = dmalloc(&c->ws.status, sizeof(int));
-    if (e == cudaSuccess) e = cudaMemset(c->ws.status, 0, sizeof(int));
+    if (e == cudaSuccess) e = alloc_workspace(c, true);
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
     if (e != cudaSuccess) {
         free_ctx(c);
@@ -364,11 +421,8 @@ emtk_status emtk_destroy(emtk_ctx *c) {
 emtk_status emtk_infer_batch(emtk_ctx *c, const emtk_request *reqs, int32_t nreq, emtk_stream stream) {
     if (!c || nreq < 0 || (nreq > 0 && !reqs)) return EMTK_ERR_ARG;
     for (int i = 0; i < nreq; ++i) {
-        const emtk_request &q = reqs[i];
-        emtk_status st = check_plane(q.d_adc, q.nwires, q.nticks, q.ld, q.d_hits, q.nhits);
+        const emtk_status st = validate_request(reqs[i]);
         if (st != EMTK_OK) return st;
-        if (q.nhits > 0 && q.d_scores == nullptr) return EMTK_ERR_ARG;
-        if ((reinterpret_cast<uintptr_t>(q.d_scores) & 3u) != 0) return EMTK_ERR_ALIGN;
     }
     c->stats.calls++;
     DeviceGuard g(c->device);

@@ -122,9 +122,18 @@ struct emtk_ctx {
     emtk::DeviceWeights w;
     emtk::Workspace ws;
     emtk_stats stats{};
+    bool owns_weights = true;  // false for a batcher lane, which shares its parent's weights
 };
 
 namespace emtk {
+
+// ---- host helpers shared by the API and the request batcher (api.cu)
+// The checks emtk_infer_batch applies to one request.
+emtk_status validate_request(const emtk_request &q);
+// A context for one batcher stream: the parent's weights and options, its own
+// workspace.  nullptr (and *st set) on failure.
+emtk_ctx *make_lane_ctx(const emtk_ctx *parent, emtk_status *st);
+void destroy_lane_ctx(emtk_ctx *c);
 
 // ---- kernels launched from the API (each returns cudaGetLastError()).
 // Interval images of every request plane: img[r] is [nwires][nint] of the

@@ -24,7 +24,8 @@ KERNELS = ("intervals", "gather", "network", "head", "convert")
 
 EXPORTED = ("emtk_default_options", "emtk_create", "emtk_destroy", "emtk_infer", "emtk_infer_batch",
             "emtk_extract_patches", "emtk_infer_patches", "emtk_check", "emtk_get_stats",
-            "emtk_status_string", "emtk_extract_patches_static")
+            "emtk_status_string", "emtk_extract_patches_static", "emtk_batcher_create", "emtk_batcher_submit",
+            "emtk_batcher_wait", "emtk_batcher_stats", "emtk_batcher_destroy")
 EMTK_STATIC_SCRATCH_BYTES = 4 << 20
 
 _vp = ctypes.c_void_p
@@ -87,6 +88,15 @@ def load_library(path: str | None = None):
     lib.emtk_extract_patches_static.argtypes = [_vp, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64, _vp,
                                                 ctypes.c_int32, _vp, ctypes.c_int, _vp]
     lib.emtk_extract_patches_static.restype = ctypes.c_int
+    lib.emtk_batcher_create.argtypes = [_vp, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64, ctypes.POINTER(_vp)]
+    lib.emtk_batcher_submit.argtypes = [_vp, ctypes.POINTER(emtk_request), ctypes.POINTER(ctypes.c_uint64)]
+    lib.emtk_batcher_wait.argtypes = [_vp, ctypes.c_uint64, ctypes.c_int64]
+    lib.emtk_batcher_stats.argtypes = [_vp, ctypes.POINTER(ctypes.c_int64), ctypes.POINTER(ctypes.c_int64),
+                                       ctypes.POINTER(ctypes.c_int64)]
+    lib.emtk_batcher_destroy.argtypes = [_vp]
+    for name in ("emtk_batcher_create", "emtk_batcher_submit", "emtk_batcher_wait", "emtk_batcher_stats",
+                 "emtk_batcher_destroy"):
+        getattr(lib, name).restype = ctypes.c_int
     lib.emtk_status_string.argtypes = [ctypes.c_int]
     lib.emtk_status_string.restype = ctypes.c_char_p
     for name in ("emtk_create", "emtk_destroy", "emtk_infer", "emtk_infer_batch", "emtk_extract_patches",
@@ -219,3 +229,37 @@ def emtk_get_stats(ctx) -> dict:
     _check(load_library().emtk_get_stats(ctx, ctypes.byref(s)), "emtk_get_stats")
     return dict(calls=s.calls, hits=s.hits, launches=s.launches, chunks=s.chunks, batch_hist=list(s.batch_hist),
                 kernel_launches=dict(zip(KERNELS, s.kernel_launches)), kernel_ms=dict(zip(KERNELS, s.kernel_ms)))
+
+
+# ------------------------------------------------------------------ batcher
+def emtk_batcher_create(ctx, nstreams: int = 4, max_hits: int = 65536, max_delay_us: int = 200):
+    """Request batcher over `ctx` (see include/emtk.h).  Returns a handle (int)."""
+    out = _vp()
+    _check(load_library().emtk_batcher_create(ctx, int(nstreams), int(max_hits), int(max_delay_us),
+                                              ctypes.byref(out)), "emtk_batcher_create")
+    return out.value
+
+
+def emtk_batcher_submit(b, adc, nticks: int, hits, scores) -> int:
+    """Queues one request (a plane, its hits and its output); returns its ticket.  The tensors
+    must stay alive and unchanged until emtk_batcher_wait has returned for the ticket."""
+    req = make_requests([(adc, nticks, hits, scores)])
+    t = ctypes.c_uint64()
+    _check(load_library().emtk_batcher_submit(b, req, ctypes.byref(t)), "emtk_batcher_submit")
+    return t.value
+
+
+def emtk_batcher_wait(b, ticket: int, timeout_ms: int = -1) -> int:
+    """Blocks until the ticket's scores are complete; returns the status (EMTK_ERR_TIMEOUT when
+    timeout_ms ran out first, without consuming the ticket)."""
+    return load_library().emtk_batcher_wait(b, int(ticket), int(timeout_ms))
+
+
+def emtk_batcher_stats(b) -> dict:
+    n = [ctypes.c_int64() for _ in range(3)]
+    _check(load_library().emtk_batcher_stats(b, *[ctypes.byref(x) for x in n]), "emtk_batcher_stats")
+    return dict(batches=n[0].value, requests=n[1].value, hits=n[2].value)
+
+
+def emtk_batcher_destroy(b) -> None:
+    _check(load_library().emtk_batcher_destroy(b), "emtk_batcher_destroy")

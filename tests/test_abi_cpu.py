@@ -107,3 +107,17 @@ def test_create_without_gpu_reports_cuda_error(lib):
 def test_missing_library_fails_loudly(tmp_path):
     with pytest.raises(RuntimeError, match="no CPU fallback"):
         emtk.load_library(str(tmp_path / "libemtk.so"))
+
+
+def test_batcher_argument_errors_without_device(lib):
+    """The batcher rejects null handles and bad sizes before touching a device."""
+    out = ctypes.c_void_p()
+    assert lib.emtk_batcher_create(None, 1, 1024, 100, ctypes.byref(out)) == emtk.EMTK_ERR_ARG
+    assert out.value is None
+    t = ctypes.c_uint64(7)
+    req = emtk.emtk_request()
+    assert lib.emtk_batcher_submit(None, ctypes.byref(req), ctypes.byref(t)) == emtk.EMTK_ERR_ARG
+    assert t.value == 0
+    assert lib.emtk_batcher_wait(None, 1, 0) == emtk.EMTK_ERR_ARG
+    assert lib.emtk_batcher_stats(None, None, None, None) == emtk.EMTK_ERR_ARG
+    assert lib.emtk_batcher_destroy(None) == emtk.EMTK_OK
