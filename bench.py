@@ -175,7 +175,7 @@ def main():
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="emtk", choices=["emtk", "reference"])
-    ap.add_argument("--workload", default="full_event", choices=["full_event", "apa", "service"])
+    ap.add_argument("--workload", default="full_event", choices=["full_event", "apa", "service", "sweep"])
     ap.add_argument("--clients", type=int, default=64, help="service workload: client threads (one event each)")
     ap.add_argument("--streams", type=int, default=8, help="service workload: batcher streams")
     ap.add_argument("--max-delay-us", type=int, default=500, help="service workload: batcher delay")
@@ -193,6 +193,8 @@ def main():
         return run_reference(args, rank, world)
     if args.workload == "service":
         return run_service(args, rank, world, local_rank)
+    if args.workload == "sweep":
+        return run_sweep(args, rank, world, local_rank)
 
     import torch
     torch.cuda.set_device(local_rank)
@@ -456,6 +458,52 @@ def run_service(args, rank, world, local_rank):
            "batches": {"count": batches, "mean_hits": (s1["hits"] - s0["hits"]) / max(1, batches),
                        "mean_requests": (s1["requests"] - s0["requests"]) / max(1, batches)},
            "timing": "host wall clock over the timed steps (a service metric); inputs resident on the device"}
+    if rank == 0:
+        print(json.dumps(out))
+
+
+def run_sweep(args, rank, world, local_rank):
+    """Inference-only batch sweep: pre-cut fp32 patches (70% zeros, else
+    lognormal(2, 1)) through emtk_infer_patches at batch sizes 256 ... 65,536
+    and the paper's 235, 1,693 and 5,358, bf16 and fp32 paths.  Per point:
+    CUDA events around `steps` calls on the stream, inputs resident, after
+    `warmup` calls."""
+    import torch
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    from paper_2009_04509_gb300 import emtk
+    weights = synth.he_normal_weights(0)
+    sizes = [235, 256, 1024, 1693, 4096, 5358, 16384, 65536]
+    x_all = torch.from_numpy(synth.inference_patches(max(sizes), seed=rank)).to(dev)
+    sc = torch.empty((max(sizes), 4), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+    table = []
+    for prec in ("bf16", "fp32"):
+        ctx = emtk.emtk_create(weights, precision=prec, device=local_rank)
+        for n in sizes:
+            x = x_all[:n]
+            for _ in range(max(3, args.warmup)):
+                emtk.emtk_infer_patches(ctx, x, sc[:n], stream)
+            steps = max(3, min(args.steps, 200 if n <= 4096 else 30 if prec == "bf16" else 5))
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            for _ in range(steps):
+                emtk.emtk_infer_patches(ctx, x, sc[:n], stream)
+            b.record(stream)
+            torch.cuda.synchronize()
+            assert emtk.emtk_check(ctx, stream) == emtk.EMTK_OK
+            ms = a.elapsed_time(b) / steps
+            table.append({"precision": prec, "batch": n, "ms_per_batch": ms, "hits_per_s": n / (ms / 1e3),
+                          "tflops": n * FLOP_PER_HIT / (ms / 1e3) / 1e12})
+        emtk.emtk_destroy(ctx)
+    best = max(r["hits_per_s"] for r in table if r["precision"] == "bf16")
+    out = {"metric": "inference-only batch sweep: patches/s of emtk_infer_patches per batch size", "value": best,
+           "unit": "hits/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": None, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+           "dtype": "bf16 and fp32", "data": "synthetic (pre-cut patches, 70% zeros, lognormal(2,1))",
+           "config": {"workload": "pre-cut 48x48 fp32 patches, batch sizes " + ", ".join(map(str, sizes)),
+                      "includes": "fp32 -> 16-bit patch conversion (16-bit paths), network, heads"},
+           "points": table}
     if rank == 0:
         print(json.dumps(out))
 

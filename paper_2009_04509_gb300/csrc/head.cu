@@ -11,6 +11,7 @@ namespace emtk {
 namespace {
 
 constexpr int kThreadsHead = 128;
+constexpr int kManyRows = 4;  // above this many partial rows per hit, reduce them with a warp per hit
 
 __global__ void __launch_bounds__(kThreadsHead) head_kernel(const float *__restrict__ partials, int splits, int G,
                                                            int n_pad, int32_t n, const float *__restrict__ fc1_b,
@@ -100,11 +101,123 @@ __global__ void __launch_bounds__(kThreadsHead) head_kernel(const float *__restr
     }
 }
 
+// The same tail when a hit has many partial rows (a small launch, whose
+// tiles are split over many CTAs): one warp per hit sums the rows, lane l
+// taking dense-1 outputs 4l .. 4l+3 of every row (512 contiguous bytes per
+// row), and writes bias + ReLU to shared memory; then one thread per hit
+// finishes as above.  32 hits per block.
+constexpr int kHitsRows = 32;
+constexpr int kThreadsRows = 256;
+constexpr int kH1Stride = kN1 + 1;  // shared h1 rows padded: thread t reads row t conflict-free
+
+__global__ void __launch_bounds__(kThreadsRows) head_rows_kernel(const float *__restrict__ partials, int splits,
+                                                                int G, int n_pad, int32_t n,
+                                                                const float *__restrict__ fc1_b,
+                                                                const float *__restrict__ fc2_w,
+                                                                const float *__restrict__ fc2_b,
+                                                                const float *__restrict__ cls_w,
+                                                                const float *__restrict__ cls_b,
+                                                                const float *__restrict__ mic_w,
+                                                                const float *__restrict__ mic_b, float *const *dest,
+                                                                int debug_logits) {
+    __shared__ float h1s[kHitsRows * kH1Stride];
+    __shared__ __align__(16) float w2[kN1][kN2];
+    __shared__ __align__(16) float wc[kN2][kNC + 1];
+    __shared__ float b2[kN2];
+    for (int i = threadIdx.x; i < kN1 * kN2; i += blockDim.x) w2[i / kN2][i % kN2] = fc2_w[i];
+    for (int i = threadIdx.x; i < kN2 * kNC; i += blockDim.x) wc[i / kNC][i % kNC] = cls_w[i];
+    for (int i = threadIdx.x; i < kN2; i += blockDim.x) {
+        wc[i][kNC] = mic_w[i];
+        b2[i] = fc2_b[i];
+    }
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t h0 = (int64_t)blockIdx.x * kHitsRows;
+    const int64_t row_stride = (int64_t)n_pad * kN1 / 4;  // float4s between partial rows
+    const float4 bb = reinterpret_cast<const float4 *>(fc1_b)[lane];
+    for (int j = warp; j < kHitsRows; j += kThreadsRows / 32) {
+        const int64_t h = h0 + j;
+        if (h >= n) break;
+        int rows = splits;
+        if (G > 0) {
+            const int64_t units = (int64_t)((n + 127) / 128) * kQuads;
+            const int64_t tile = h >> 7;
+            rows = cta_of_unit(tile * kQuads + kQuads - 1, units, G) - cta_of_unit(tile * kQuads, units, G) + 1;
+        }
+        const float4 *p = reinterpret_cast<const float4 *>(partials + h * kN1) + lane;
+        float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
+        for (int r = 0; r < rows; ++r) {  // rows in order: the same sum as head_kernel
+            const float4 v = p[r * row_stride];
+            a.x += v.x;
+            a.y += v.y;
+            a.z += v.z;
+            a.w += v.w;
+        }
+        float *o = h1s + j * kH1Stride + 4 * lane;
+        o[0] = fmaxf(a.x + bb.x, 0.f);
+        o[1] = fmaxf(a.y + bb.y, 0.f);
+        o[2] = fmaxf(a.z + bb.z, 0.f);
+        o[3] = fmaxf(a.w + bb.w, 0.f);
+    }
+    __syncthreads();
+    if (threadIdx.x >= kHitsRows) return;
+    const int64_t h = h0 + threadIdx.x;
+    if (h >= n) return;
+    const float *h1 = h1s + threadIdx.x * kH1Stride;
+    float h2[kN2];
+#pragma unroll
+    for (int j = 0; j < kN2; ++j) h2[j] = b2[j];
+    for (int k = 0; k < kN1; ++k) {
+        const float x = h1[k];
+        const float4 *wr = reinterpret_cast<const float4 *>(&w2[k][0]);
+#pragma unroll
+        for (int q = 0; q < kN2 / 4; ++q) {
+            const float4 wv = wr[q];
+            h2[4 * q + 0] = fmaf(x, wv.x, h2[4 * q + 0]);
+            h2[4 * q + 1] = fmaf(x, wv.y, h2[4 * q + 1]);
+            h2[4 * q + 2] = fmaf(x, wv.z, h2[4 * q + 2]);
+            h2[4 * q + 3] = fmaf(x, wv.w, h2[4 * q + 3]);
+        }
+    }
+    float z[kNC + 1] = {cls_b[0], cls_b[1], cls_b[2], mic_b[0]};
+#pragma unroll
+    for (int j = 0; j < kN2; ++j) {
+        const float v = fmaxf(h2[j], 0.f);
+        const float4 wv = *reinterpret_cast<const float4 *>(&wc[j][0]);
+        z[0] = fmaf(v, wv.x, z[0]);
+        z[1] = fmaf(v, wv.y, z[1]);
+        z[2] = fmaf(v, wv.z, z[2]);
+        z[3] = fmaf(v, wv.w, z[3]);
+    }
+    const float m = fmaxf(fmaxf(z[0], z[1]), z[2]);
+    const float e0 = expf(z[0] - m), e1 = expf(z[1] - m), e2 = expf(z[2] - m);
+    const float sum = e0 + e1 + e2;
+    float *out = dest[h];
+    out[0] = e0 / sum;
+    out[1] = e1 / sum;
+    out[2] = e2 / sum;
+    out[3] = 1.0f / (1.0f + expf(-z[kNC]));
+    if (debug_logits) {
+        out[4] = z[0];
+        out[5] = z[1];
+        out[6] = z[2];
+        out[7] = z[3];
+    }
+}
+
 }  // namespace
 
 cudaError_t launch_head(const DeviceWeights &w, const float *partials, int splits, int G, int n_pad, int32_t n,
                         float *const *dest, int debug_logits, cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
+    // most partial rows a hit has: many when a small launch spreads each tile over many CTAs
+    const int rows = G > 0 ? streamk_partial_rows(n, G) : splits;
+    if (rows > kManyRows) {
+        head_rows_kernel<<<(n + kHitsRows - 1) / kHitsRows, kThreadsRows, 0, s>>>(
+            partials, splits, G, n_pad, n, w.fc1_b, w.fc2_w, w.fc2_b, w.cls_w, w.cls_b, w.mic_w, w.mic_b, dest,
+            debug_logits);
+        return cudaGetLastError();
+    }
     head_kernel<<<(n + kThreadsHead - 1) / kThreadsHead, kThreadsHead, 0, s>>>(
         partials, splits, G, n_pad, n, w.fc1_b, w.fc2_w, w.fc2_b, w.cls_w, w.cls_b, w.mic_w, w.mic_b, dest,
         debug_logits);
