@@ -458,6 +458,12 @@ def run_service(args, rank, world, local_rank):
            "batches": {"count": batches, "mean_hits": (s1["hits"] - s0["hits"]) / max(1, batches),
                        "mean_requests": (s1["requests"] - s0["requests"]) / max(1, batches)},
            "timing": "host wall clock over the timed steps (a service metric); inputs resident on the device"}
+    # the paper's scale-out model (Sec. 3.3) with its CPU job and this throughput as t_gpu
+    from paper_2009_04509_gb300 import sonic
+    job = sonic.gb300_job(out["value"])
+    out["sonic_model"] = {"t_gpu_s_per_55k_inferences": job.t_gpu, "cpu_jobs_per_gpu": sonic.cpu_per_gpu(job),
+                          "paper_cpu_jobs_per_gpu_model": sonic.cpu_per_gpu(sonic.paper_job()),
+                          "paper_measured": "about 68 CPU processes per T4 (270 on 4 GPUs)"}
     if rank == 0:
         print(json.dumps(out))
 
