@@ -64,6 +64,8 @@ def _bind(path: str):
     lib.or_heads.argtypes = [f64p, ctypes.c_int, ctypes.c_double, f64p]
     lib.or_round_bf16.argtypes = [f32p, ctypes.POINTER(ctypes.c_uint16), ctypes.c_long]
     lib.or_round_fp16.argtypes = [f32p, f32p, ctypes.c_long]
+    lib.or_round_e4m3.argtypes = [f32p, f32p, ctypes.c_long]
+    lib.or_set_fp8_scales.argtypes = [ctypes.c_double, ctypes.c_double]
     lib.or_set_threads.argtypes = [ctypes.c_int]
     lib.or_max_threads.restype = ctypes.c_int
     return lib
@@ -107,16 +109,20 @@ def extract_patches(adc, nticks, hits, psize: int = PATCH, ds: int = DOWNSAMPLE,
 _WKEYS = ("conv_w", "conv_b", "fc1_w", "fc1_b", "fc2_w", "fc2_b", "cls_w", "cls_b", "mic_w", "mic_b")
 
 
-_EMULATE = {None: 0, "bf16": 1, "fp16": 2}
+_EMULATE = {None: 0, "bf16": 1, "fp16": 2, "fp8": 3}
 
 
 def forward(patches, weights: dict, dims: dict | None = None, emulate: str | None = None,
-            threads: int | None = None, lib=None):
+            threads: int | None = None, lib=None, fp8_scales: tuple = (1.0, 1.0)):
     """Sec. 2.2 network on [n][P][P] float32 patches.  Returns (logits, scores),
     each [n][NC+1] float64: softmax classes (track, em, none) then Michel.
     ``emulate`` = "bf16" or "fp16" rounds the operands of the conv and of
-    dense-1 to that format first (a diagnostic reference for 16-bit paths)."""
+    dense-1 to that format first (a diagnostic reference for 16-bit paths);
+    "fp8" rounds the conv operands to bf16 and the dense-1 operands to e4m3,
+    as e4m3(a * s_a) / s_a and e4m3(w * s_w) / s_w with (s_a, s_w) =
+    ``fp8_scales``."""
     lib = lib or load()
+    lib.or_set_fp8_scales(float(fp8_scales[0]), float(fp8_scales[1]))
     d = dict(EMTK_DIMS if dims is None else dims)
     patches = _c(patches, np.float32).reshape(-1, d["P"], d["P"])
     n = patches.shape[0]
@@ -186,6 +192,16 @@ def round_fp16(x, lib=None):
     x = _c(x, np.float32)
     out = np.zeros(x.shape, np.float32)
     lib.or_round_fp16(_p(x, ctypes.c_float), _p(out, ctypes.c_float), x.size)
+    return out
+
+
+def round_e4m3(x, lib=None):
+    """Round float32 values to FP8 E4M3 (nearest, ties to even, saturating at
+    +-448); returns float32."""
+    lib = lib or load()
+    x = _c(x, np.float32)
+    out = np.zeros(x.shape, np.float32)
+    lib.or_round_e4m3(_p(x, ctypes.c_float), _p(out, ctypes.c_float), x.size)
     return out
 
 

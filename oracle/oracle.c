@@ -89,16 +89,60 @@ static float round_fp16_f(float x)
     return copysignf(r, x);
 }
 
+/* Round a finite float to the nearest FP8 E4M3 value (sign, 4 exponent bits
+ * with bias 7, 3 mantissa bits; no infinities), ties to even, gradual
+ * underflow below 2^-6 (spacing 2^-9), saturating at +-448 (the largest
+ * finite value); returned as a float. */
+static float round_e4m3_f(float x)
+{
+    if (x == 0.0f || isnan(x))
+        return x;
+    const float a = fabsf(x);
+    int e;
+    frexpf(a, &e);              /* a in [2^(e-1), 2^e) */
+    int qexp = e - 4;           /* 4 significant bits */
+    if (qexp < -9)
+        qexp = -9;              /* subnormal spacing 2^-9 */
+    const float q = ldexpf(1.0f, qexp);
+    float r = rintf(a / q) * q; /* a / q is exact: q is a power of two */
+    if (r > 448.0f)
+        r = 448.0f;
+    return copysignf(r, x);
+}
+
+void or_round_e4m3(const float *in, float *out, long n)
+{
+    for (long i = 0; i < n; ++i)
+        out[i] = round_e4m3_f(in[i]);
+}
+
+/* Power-of-two scales of the fp8 emulation: dense-1 activations are rounded
+ * as e4m3(a * act_scale) / act_scale, its weights as e4m3(w * w_scale) /
+ * w_scale. */
+static double fp8_act_scale = 1.0, fp8_w_scale = 1.0;
+
+void or_set_fp8_scales(double act_scale, double w_scale)
+{
+    fp8_act_scale = act_scale;
+    fp8_w_scale = w_scale;
+}
+
 void or_round_fp16(const float *in, float *out, long n)
 {
     for (long i = 0; i < n; ++i)
         out[i] = round_fp16_f(in[i]);
 }
 
-/* emulation modes: 0 none, 1 bf16, 2 fp16 */
+/* emulation modes: 0 none, 1 bf16, 2 fp16, 3 fp8 (bf16 conv operands, e4m3
+ * dense-1 operands); round_mode covers the 16-bit roundings */
 static float round_mode(float x, int mode)
 {
-    return mode == 1 ? round_bf16_f(x) : mode == 2 ? round_fp16_f(x) : x;
+    return (mode == 1 || mode == 3) ? round_bf16_f(x) : mode == 2 ? round_fp16_f(x) : x;
+}
+
+static float round_scaled_e4m3(float x, double scale)
+{
+    return (float)((double)round_e4m3_f((float)((double)x * scale)) / scale);
 }
 
 void or_round_bf16(const float *in, uint16_t *out, long n)
@@ -247,7 +291,9 @@ void or_heads(const double *logits, int NC, double logit_m, double *scores)
  * header comment, fp32.  Outputs (each [n][NC+1], double): the logits (NC
  * class logits then the Michel logit) and the scores (softmax then sigmoid).
  * emulate = 1 (bf16) or 2 (fp16) rounds patch, conv weights, post-ReLU conv
- * outputs and dense-1 weights to that format before use; 0 rounds nothing. */
+ * outputs and dense-1 weights to that format before use; 3 (fp8) rounds
+ * patch and conv weights to bf16 and the post-ReLU conv outputs and dense-1
+ * weights to e4m3 with the scales of or_set_fp8_scales; 0 rounds nothing. */
 int or_forward(const or_dims *d, const float *patches, long n,
                const float *conv_w, const float *conv_b,
                const float *fc1_w, const float *fc1_b,
@@ -260,7 +306,7 @@ int or_forward(const or_dims *d, const float *patches, long n,
         return OR_ERR_ARG;
     const int P = d->P, R = d->R, F = d->F, N1 = d->N1, N2 = d->N2, NC = d->NC;
     if (P <= 0 || R <= 0 || R > P || F <= 0 || N1 <= 0 || N2 <= 0 || NC <= 0 ||
-        emulate < 0 || emulate > 2)
+        emulate < 0 || emulate > 3)
         return OR_ERR_ARG;
     if (n == 0)
         return OR_OK;
@@ -289,7 +335,7 @@ int or_forward(const or_dims *d, const float *patches, long n,
             return OR_ERR_OOM;
         }
         for (long i = 0; i < K1 * N1; ++i)
-            w1[i] = round_mode(fc1_w[i], emulate);
+            w1[i] = emulate == 3 ? round_scaled_e4m3(fc1_w[i], fp8_w_scale) : round_mode(fc1_w[i], emulate);
         W1 = w1;
     }
 
@@ -311,7 +357,10 @@ int or_forward(const or_dims *d, const float *patches, long n,
                 for (int i = 0; i < P * P; ++i)
                     img[i] = (double)round_mode(p[i], emulate);
                 or_conv_relu(img, P, cw, cb, R, F, act);
-                if (emulate)
+                if (emulate == 3)
+                    for (long k = 0; k < K1; ++k)
+                        act[k] = (double)round_scaled_e4m3((float)act[k], fp8_act_scale);
+                else if (emulate)
                     for (long k = 0; k < K1; ++k)
                         act[k] = (double)round_mode((float)act[k], emulate);
                 or_dense(act, K1, W1, fc1_b, N1, 1, h1);

@@ -288,10 +288,55 @@ def pin_transmit_volume(lib):
     assert abs(bits / 1e9 - FACTS["transmit_gbit_per_event"]) < 0.06
 
 
+# ------------------------------------------------------------- fp8 (e4m3)
+def e4m3_table():
+    """Every finite FP8 E4M3 value, from the format's definition: sign, 4-bit
+    exponent (bias 7), 3-bit mantissa; exponent 0 is subnormal; the code with
+    all exponent and mantissa bits set is NaN, so 448 is the largest."""
+    vals = set()
+    for e in range(16):
+        for m in range(8):
+            if e == 15 and m == 7:
+                continue
+            v = (m / 8.0) * 2.0 ** -6 if e == 0 else (1 + m / 8.0) * 2.0 ** (e - 7)
+            vals.add(v)
+            vals.add(-v)
+    return np.array(sorted(vals))
+
+
+def test_e4m3_table_facts():
+    t = e4m3_table()
+    assert t.max() == 448.0 and np.min(t[t > 0]) == 2.0 ** -9
+    assert len(t) == 2 * 127 - 1  # 127 non-negative finite codes each side, +-0 merged
+
+
+def pin_e4m3_rounding(lib):
+    t = e4m3_table()
+    # representable values map to themselves
+    assert np.array_equal(oracle.round_e4m3(t.astype(np.float32), lib=lib), t.astype(np.float32))
+    rng = np.random.default_rng(7)
+    x = np.concatenate([rng.standard_normal(20000) * s for s in (0.003, 0.1, 3.0, 100.0)]).astype(np.float32)
+    got = oracle.round_e4m3(x, lib=lib).astype(np.float64)
+    xs = np.clip(x.astype(np.float64), -448.0, 448.0)
+    dist = np.abs(t[None, :] - xs[:, None])
+    best = dist.min(1)
+    assert np.allclose(np.abs(got - xs), best, rtol=0, atol=0)  # a nearest value
+    # ties (midpoints between neighbours) go to the even mantissa
+    pos = t[t > 0]
+    mids = ((pos[:-1] + pos[1:]) / 2).astype(np.float32)
+    r = oracle.round_e4m3(mids, lib=lib).astype(np.float64)
+    for mval, rv in zip(mids.astype(np.float64), r):
+        lo, hi = pos[pos < mval].max(), pos[pos > mval].min()
+        even = lo if int(round(lo / 2.0 ** (np.floor(np.log2(max(lo, 2.0 ** -6))) - 3))) % 2 == 0 else hi
+        assert rv == even, (mval, rv, lo, hi)
+    assert oracle.round_e4m3(np.array([1e4, -1e4], np.float32), lib=lib).tolist() == [448.0, -448.0]
+
+
+
 PINS = [pin_parameter_count, pin_conv_shape, pin_constant_plane, pin_ramps, pin_impulse,
         pin_outside_and_partial, pin_negative_ticks, pin_patches_brute_force, pin_conv_library,
         pin_dense_library, pin_heads, pin_forward_library, pin_forward_full_size, pin_zero_weights,
-        pin_flatten_order, pin_bf16_rounding, pin_fp16_rounding, pin_transmit_volume]
+        pin_flatten_order, pin_bf16_rounding, pin_fp16_rounding, pin_transmit_volume, pin_e4m3_rounding]
 
 
 @pytest.mark.parametrize("pin", PINS, ids=[p.__name__ for p in PINS])
@@ -335,6 +380,10 @@ MUTATIONS = {
                           "or_dense(h1, N1, fc2_w, fc2_b, N2, 0, h2);"),
     "flatten_chw": ("out[((long)y * Q + x) * F + f]", "out[((long)f * Q + y) * Q + x]"),
     "partial_interval_read": ("const long nint = nticks / ds;", "const long nint = (nticks + ds - 1) / ds;"),
+    "e4m3_four_mantissa_bits": ("int qexp = e - 4;           /* 4 significant bits */",
+                                "int qexp = e - 5;           /* 4 significant bits */"),
+    "e4m3_no_subnormals": ("if (qexp < -9)\n        qexp = -9;", "if (qexp < -6)\n        qexp = -6;"),
+    "e4m3_no_saturation": ("if (r > 448.0f)\n        r = 448.0f;", "if (r > 480.0f)\n        r = 480.0f;"),
     "wire_col_swap": ("v = interval_value(plane + w * ld, b, ds);",
                       "v = (w < nint && b < nwires) ? interval_value(plane + b * ld, w, ds) : 0.0f;"),
 }
@@ -362,3 +411,22 @@ def test_planted_mistakes(name, tmp_path, oracle_lib):
         except (AssertionError, ValueError, FloatingPointError):
             failed.append(pin.__name__)
     assert failed, f"planted mistake {name} passed every pin"
+
+
+def test_fp8_emulation_is_rounding_only(oracle_lib):
+    """The fp8 mode equals the plain mode on inputs whose bf16 conv operands,
+    scaled activations and scaled dense-1 weights are already e4m3 values."""
+    rng = np.random.default_rng(13)
+    d = dict(P=6, R=1, F=1, N1=4, N2=3, NC=3)
+    wt = synth.he_normal_weights(5, bias_std=0.1, dims=d)
+    wt["conv_w"][:] = 1.0
+    wt["conv_b"][:] = 0.0
+    t = e4m3_table()
+    sa, sw = 0.25, 16.0
+    wt["fc1_w"] = (rng.choice(t[np.abs(t) <= 100], wt["fc1_w"].shape) / sw).astype(np.float32)
+    x = (rng.choice(t[(t >= 0) & (t <= 200)], (4, 6, 6)) / sa).astype(np.float32)  # bf16 values too
+    a = oracle.forward(x, wt, dims=d)
+    b = oracle.forward(x, wt, dims=d, emulate="fp8", fp8_scales=(sa, sw))
+    assert np.array_equal(a[0], b[0])
+    c = oracle.forward(x * 1.1, wt, dims=d, emulate="fp8", fp8_scales=(sa, sw))  # beyond e4m3 spacing
+    assert not np.array_equal(a[0], c[0]) and np.all(np.isfinite(c[1]))
