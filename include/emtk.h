@@ -59,8 +59,17 @@ typedef enum {
  *              dense-2 and heads in fp32.
  *   EMTK_FP16: as EMTK_BF16 with IEEE fp16 operands (same tensor rate,
  *              8x finer rounding; activations above 65504 saturate).
+ *   EMTK_FP8:  the conv as EMTK_BF16; dense-1 (92,928 -> 128, Sec. 2.2)
+ *              with FP8 E4M3 operands (4 exponent bits, bias 7, 3 mantissa
+ *              bits, largest finite 448; round to nearest even, saturating
+ *              to +-448) at twice the bf16 tensor rate.  Both operands are
+ *              scaled by powers of two before rounding: activations by
+ *              s_a = 2^-4, weights by s_w, the largest power of two with
+ *              max|W1| * s_w <= 448; the fp32 sums are multiplied by
+ *              1 / (s_a s_w) before the dense-1 bias (emtk_get_fp8_scales).
+ *              Patches are bf16.
  *   EMTK_TF32: reserved; emtk_create returns EMTK_ERR_UNSUPPORTED. */
-typedef enum { EMTK_FP32 = 0, EMTK_TF32 = 1, EMTK_BF16 = 2, EMTK_FP16 = 3 } emtk_precision;
+typedef enum { EMTK_FP32 = 0, EMTK_TF32 = 1, EMTK_BF16 = 2, EMTK_FP16 = 3, EMTK_FP8 = 4 } emtk_precision;
 
 /* Element type of a patch buffer. */
 typedef enum { EMTK_PATCH_F32 = 0, EMTK_PATCH_BF16 = 1, EMTK_PATCH_F16 = 2 } emtk_patch_format;
@@ -208,6 +217,11 @@ EMTK_API emtk_status emtk_check(emtk_ctx *ctx, emtk_stream stream);
 /* Counters since creation.  In profile mode this first waits for the events
  * of every launch not yet read back. */
 EMTK_API emtk_status emtk_get_stats(emtk_ctx *ctx, emtk_stats *out);
+
+/* The dense-1 operand scales of an EMTK_FP8 context (see emtk_precision):
+ * *s_a = 2^-4 and *s_w; 1 and 1 for every other precision.  Either pointer
+ * may be NULL.  EMTK_ERR_ARG for a NULL context. */
+EMTK_API emtk_status emtk_get_fp8_scales(const emtk_ctx *ctx, float *s_a, float *s_w);
 
 /* Static English text for a status code. */
 EMTK_API const char *emtk_status_string(emtk_status s);

@@ -25,10 +25,13 @@ struct DeviceGuard {  // restores the caller's current device
     }
 };
 
-bool tensor_precision(emtk_precision p) { return p == EMTK_BF16 || p == EMTK_FP16; }
+bool tensor_precision(emtk_precision p) { return p == EMTK_BF16 || p == EMTK_FP16 || p == EMTK_FP8; }
 
+TcMode tc_mode(emtk_precision p) { return p == EMTK_FP16 ? kTcFp16 : p == EMTK_FP8 ? kTcFp8 : kTcBf16; }
+
+// EMTK_FP8 keeps the conv in bf16, so its patches are bf16
 emtk_patch_format patch_format(emtk_precision p) {
-    return p == EMTK_BF16 ? EMTK_PATCH_BF16 : p == EMTK_FP16 ? EMTK_PATCH_F16 : EMTK_PATCH_F32;
+    return (p == EMTK_BF16 || p == EMTK_FP8) ? EMTK_PATCH_BF16 : p == EMTK_FP16 ? EMTK_PATCH_F16 : EMTK_PATCH_F32;
 }
 
 size_t patch_elem_bytes(emtk_patch_format f) { return f == EMTK_PATCH_F32 ? 4 : 2; }
@@ -164,7 +167,7 @@ emtk_status run_network(emtk_ctx *c, const void *patches, const HitDesc *desc, i
         G = c->sm_count;
         while (G > 1 && streamk_partial_rows(n, G) > max_splits) G /= 2;
         Prof prof(c, EMTK_KERNEL_NETWORK, s);
-        e = launch_cnn_tc(c->w, patches, desc, c->opt.precision == EMTK_FP16, n, G, c->ws.partials, n_pad,
+        e = launch_cnn_tc(c->w, patches, desc, tc_mode(c->opt.precision), n, G, c->ws.partials, n_pad,
                           c->ws.status, c->opt.wait_timeout_ns, c->opt.debug_stall, s);
     } else {
         splits = choose_splits_fp32(n, c->sm_count, max_splits);
@@ -359,7 +362,7 @@ emtk_status emtk_create(const emtk_weights *w, const emtk_options *opt, int devi
     emtk_default_options(&o);
     if (opt) o = *opt;
     if (o.precision != EMTK_FP32 && o.precision != EMTK_TF32 && o.precision != EMTK_BF16 &&
-        o.precision != EMTK_FP16)
+        o.precision != EMTK_FP16 && o.precision != EMTK_FP8)
         return EMTK_ERR_ARG;
     if (o.max_hits <= 0 || o.wait_timeout_ns <= 0 || (o.debug_logits != 0 && o.debug_logits != 1) ||
         (o.profile != 0 && o.profile != 1) || (o.debug_stall != 0 && o.debug_stall != 1))
@@ -393,7 +396,7 @@ emtk_status emtk_create(const emtk_weights *w, const emtk_options *opt, int devi
     if (e == cudaSuccess) e = upload(&d.mic_b, w->mic_b, 1);
     if (e == cudaSuccess) {
         if (tensor_precision(o.precision)) {
-            e = prepare_tc_weights(d, *w, o.precision == EMTK_FP16);
+            e = prepare_tc_weights(d, *w, tc_mode(o.precision));
             if (e == cudaSuccess) e = init_tc_kernel_attrs();
         } else {
             e = upload(&d.fc1_w, w->fc1_w, (size_t)kFc1In * kN1);
@@ -525,6 +528,14 @@ emtk_status emtk_get_stats(emtk_ctx *c, emtk_stats *out) {
         drain_events(c);
     }
     *out = c->stats;
+    return EMTK_OK;
+}
+
+emtk_status emtk_get_fp8_scales(const emtk_ctx *c, float *s_a, float *s_w) {
+    if (!c) return EMTK_ERR_ARG;
+    const bool f8 = c->opt.precision == EMTK_FP8;
+    if (s_a) *s_a = f8 ? 1.0f / (c->w.fc1_scale * c->w.fc1_w_scale) : 1.0f;
+    if (s_w) *s_w = f8 ? c->w.fc1_w_scale : 1.0f;
     return EMTK_OK;
 }
 

@@ -1,34 +1,38 @@
-// 16-bit network path on the sm_103a tensor cores (EMTK_BF16 / EMTK_FP16):
+// Tensor-core network path on sm_103a (EMTK_BF16 / EMTK_FP16 / EMTK_FP8):
 // the conv 5x5x48 + ReLU (Sec. 2.2) fused into dense-1 (92,928 -> 128), so
 // the 92,928 conv activations of a hit never leave the SM.
 //
-// One CTA = 128 hits (one TMEM lane each) x one segment of the dense-1 input
-// dimension.  Conv positions p = y*44 + x are walked in quads (4 positions
-// of one row; the dense-1 input index is p*48 + c, the paper's channels-last
-// flatten), and each quad is two position pairs (x, x+1):
+// Work units are (tile of 128 hits, quad of 4 conv positions of one output
+// row): 484 quads per tile, each supplying 192 consecutive dense-1 inputs
+// (input index = position * 48 + filter, the channels-last flatten).  One
+// persistent CTA per SM takes a contiguous range of units (stream-K), across
+// tile boundaries; a quad is two position pairs (x, x+1):
 //   builder warps   write, per hit, the 5 x 6 window of a pair (30 taps) and
 //                   two bias taps of 1.0 as one 32-wide im2col row into a
 //                   swizzled shared-memory tile (one 128-byte row per hit and
-//                   quad);
-//   MMA warp        conv MMA  D[128 x 96] = A_smem[128 x 32] * Bpair[32 x 96]:
-//                   columns 0-47 are the 48 filters at x (tap column 5 has a
-//                   zero weight), columns 48-95 the filters at x+1 (tap
-//                   column 0 zero); the conv bias rides on the bias taps;
-//   epilogue warps  ReLU + round the 128 x 96 conv tile to 16 bit, written
-//                   back into TMEM over it;
-//   MMA warp        dense-1  ACC[128 x 128] += A_tmem[128 x 96] * W1[96 x 128],
-//                   W1 streamed by TMA through a 3-stage ring (one quad, 48 KB,
-//                   per stage, 128-byte swizzle).
-// The MMA stream alternates [conv of quad q (2 pairs)] [dense-1 of quad q-1
-// (12 MMAs into one accumulator)], which keeps the tensor pipe busy while a
-// conv tile makes its round trip through the epilogue.  Every wait is
-// bounded: on timeout the CTA raises an abort flag, sets bit 0 of the status
-// word, waits for its in-flight copies and MMAs, frees TMEM and returns.
+//                   quad), reading the window straight from the hit's plane
+//                   image;
+//   conv issuer     D[128 x 96] = A_smem[128 x 32] * Bpair[32 x 96] (16 bit):
+//                   columns 0-47 are the 48 filters at x, 48-95 at x+1; the
+//                   conv bias rides on the bias taps;
+//   epilogue warps  ReLU + round the 128 x 96 conv tile (to 16 bit, or to
+//                   e4m3: there the conv weights and bias are scaled by
+//                   kFp8ActScale, a power of two, so the tile is already the
+//                   scaled activation), written back into TMEM over it;
+//   dense-1 issuer  ACC[128 x 128] += A_tmem[128 x 96] * W1[96 x 128], W1
+//                   streamed by TMA through a 3-stage ring (one quad per
+//                   stage: 48 KB of 16-bit or 24 KB of e4m3 weights);
+//   at a tile's end the epilogue drains ACC to the CTA's partial-sum row.
+// Every wait is bounded: on timeout the CTA raises an abort flag, sets bit 0
+// of the status word, waits for its in-flight copies and MMAs, frees TMEM
+// and returns.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
+#include <cuda_fp8.h>
 #include <cudaTypedefs.h>
 
+#include <cmath>
 #include <vector>
 
 #include "emtk_internal.h"
@@ -45,8 +49,7 @@ namespace {
 constexpr int kThreadsTC = 352;  // 11 warps
 constexpr int kTmaWarp = 0;
 constexpr int kConvWarp = 1;
-constexpr int kFc1Warp = 3;
-constexpr int kEpiWarp0 = 4;     // warps 4-7: epilogue, TMEM lane quarter warp mod 4
+constexpr int kFc1Warp = 3;      // warps 4-7: epilogue, TMEM lane quarter warp mod 4
 __host__ __device__ constexpr int builder_index(int warp) {  // warps 2, 8, 9, 10 -> row blocks 0-3
     return warp == 2 ? 0 : warp >= 8 ? warp - 7 : -1;
 }
@@ -68,6 +71,12 @@ constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kAccCol = 0;                              // dense-1 accumulator, 128 fp32 columns
 constexpr uint32_t kSlotCol0 = 128;                          // conv fp32 tile of a pair, then its activations
 constexpr uint32_t kSlotCols = kPairN;
+// EMTK_FP8: dense-1 operands in e4m3.  A W1 box is 64 inputs x 128 outputs of
+// one byte (64-byte swizzle), a stage 3 boxes; activations are scaled by
+// kFp8ActScale (a power of two) before rounding.
+constexpr int kW1BoxBytesF8 = kW1Box * kN1;                  // 8192
+constexpr int kW1StageBytesF8 = kBoxesPerStage * kW1BoxBytesF8;  // 24576
+constexpr float kFp8ActScale = 0.0625f;
 
 constexpr int kOffW1 = 0;
 constexpr int kOffIm = kOffW1 + kW1Stages * kW1StageBytes;
@@ -192,6 +201,15 @@ __device__ __forceinline__ void mma_ss(uint32_t d, uint64_t adesc, uint64_t bdes
         "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accum)
         : "memory");
 }
+// D[tmem] (+)= A[tmem] * B[smem desc], kind::f8f6f4 (e4m3 x e4m3), one CTA.
+__device__ __forceinline__ void mma_ts_f8(uint32_t d, uint32_t a, uint64_t bdesc, uint32_t idesc, uint32_t accum) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d),
+        "r"(a), "l"(bdesc), "r"(idesc), "r"(accum)
+        : "memory");
+}
 __device__ __forceinline__ void mma_commit(uint32_t bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
                  : "memory");
@@ -246,7 +264,22 @@ __device__ __forceinline__ uint32_t relu_pack(uint32_t lo, uint32_t hi) {
     return d;
 }
 
+// ReLU of four fp32 values as four e4m3 bytes of one word, element 0 in the
+// lowest byte; satfinite clamps to 448.
+__device__ __forceinline__ uint32_t relu_e4m3x4(uint32_t v0, uint32_t v1, uint32_t v2, uint32_t v3) {
+    uint32_t r;
+    asm("{\n\t.reg .b16 lo, hi;\n\t"
+        "cvt.rn.satfinite.relu.e4m3x2.f32 lo, %2, %1;\n\t"
+        "cvt.rn.satfinite.relu.e4m3x2.f32 hi, %4, %3;\n\t"
+        "mov.b32 %0, {lo, hi};\n\t}"
+        : "=r"(r)
+        : "f"(__uint_as_float(v0)), "f"(__uint_as_float(v1)), "f"(__uint_as_float(v2)), "f"(__uint_as_float(v3)));
+    return r;
+}
+
 // Instruction descriptor, kind::f16: fp32 accumulate, both operands K-major.
+// With fp16 = true the format codes (0) are also those of e4m3 x e4m3 for
+// kind::f8f6f4.
 __host__ __device__ constexpr uint32_t make_idesc(int M, int N, bool fp16) {
     return (1u << 4) | ((fp16 ? 0u : 1u) << 7) | ((fp16 ? 0u : 1u) << 10) | ((uint32_t)(N >> 3) << 17) |
            ((uint32_t)(M >> 4) << 24);
@@ -257,6 +290,11 @@ __host__ __device__ constexpr uint32_t make_idesc(int M, int N, bool fp16) {
 __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
     return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
            ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+// The same for a 64-byte swizzle: 64-byte rows, 8-row groups 512 bytes apart.
+__device__ __forceinline__ uint64_t sw64_desc(uint32_t saddr) {
+    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(512 >> 4) << 32) |
+           ((uint64_t)1 << 46) | ((uint64_t)4 << 61);
 }
 
 // One 48-wide row of a hit's window, 16-bit pixels packed two per word:
@@ -319,7 +357,8 @@ __device__ __forceinline__ void load_window_row_checked(const uint16_t *__restri
 }
 
 // ------------------------------------------------------------------ kernel
-template <bool FP16>
+// MODE kTcBf16, kTcFp16, or kTcFp8 (bf16 conv, e4m3 dense-1).
+template <int MODE>
 __global__ void __launch_bounds__(kThreadsTC, 1)
     cnn_tc_kernel(const __grid_constant__ CUtensorMap tmap_w1, const uint16_t *__restrict__ src,
                   const HitDesc *__restrict__ desc, int n,
@@ -346,6 +385,10 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     const int qt0 = (int)(u0 % kW1Steps);           // quad-in-tile and tile of the first unit
     const int tile0 = (int)(u0 / kW1Steps);
     const Guard guard{abort_flag, status, (int64_t)timeout_ns};
+    constexpr bool FP16 = MODE == kTcFp16;  // 16-bit format of the conv operands
+    constexpr bool F8 = MODE == kTcFp8;     // e4m3 dense-1
+    constexpr int kStageTx = F8 ? kW1StageBytesF8 : kW1StageBytes;
+    constexpr int kBoxTx = F8 ? kW1BoxBytesF8 : kW1BoxBytes;
 
     // ---- set-up: pair conv B operand into swizzled smem, barriers, TMEM
     for (int idx = threadIdx.x; idx < kPairN * 8; idx += kThreadsTC) {
@@ -404,10 +447,10 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                     ok = false;
                     break;
                 }
-                mbar_expect_tx(bar(kBarW1Full + wj), kW1StageBytes);
+                mbar_expect_tx(bar(kBarW1Full + wj), kStageTx);
 #pragma unroll
                 for (int a = 0; a < kBoxesPerStage; ++a)
-                    tma_load_3d(sW1 + wj * kW1StageBytes + a * kW1BoxBytes, &tmap_w1, bar(kBarW1Full + wj), 0, 0,
+                    tma_load_3d(sW1 + wj * kW1StageBytes + a * kBoxTx, &tmap_w1, bar(kBarW1Full + wj), 0, 0,
                                 kBoxesPerStage * qt + a);
                 ++issued;
             }
@@ -466,7 +509,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                     mma_commit(bar(kBarImFree + ib));
                 }
             } else {
-                constexpr uint32_t idesc_fc1 = make_idesc(128, kN1, FP16);
+                constexpr uint32_t idesc_fc1 = make_idesc(128, kN1, FP16 || F8);
                 int tiles_done = 0;  // tile segments whose accumulator was handed to the epilogue
                 int qt = qt0 - 1;
                 for (int q = 0; ok && q < nq; ++q) {
@@ -488,21 +531,31 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                         break;
                     }
                     tc_fence_after();
-                    const uint64_t wdesc = sw128_desc(sW1 + wj * kW1StageBytes);
+                    // K steps of 32 bytes per row: 16 inputs (16 bit) or 32 (e4m3); a pair's 96
+                    // inputs are 6 or 3 steps, 8 TMEM columns each
+                    constexpr int kSteps = F8 ? 6 : 12;
+                    constexpr int kHalf = kSteps / 2;
+                    constexpr int kStepsPerBox = kW1Box * (F8 ? 1 : 2) / 32;
+                    const uint64_t wdesc = F8 ? sw64_desc(sW1 + wj * kW1StageBytes) : sw128_desc(sW1 + wj * kW1StageBytes);
 #pragma unroll
-                    for (int step = 0; step < 12; ++step) {  // 16-wide K steps of the quad's 192
+                    for (int step = 0; step < kSteps; ++step) {
                         // the second pair's activations are waited for only when its half begins
-                        if (step == 6) {
+                        if (step == kHalf) {
                             if (!wait_bounded(bar(kBarAct + s1), par, guard)) {
                                 ok = false;
                                 break;
                             }
                             tc_fence_after();
                         }
-                        const uint32_t a = tmem + kSlotCol0 + (uint32_t)(step < 6 ? s0 : s1) * kSlotCols + 8u * (step % 6);
-                        const uint64_t bd = wdesc + (uint64_t)(((step >> 2) * kW1BoxBytes + (step & 3) * 32) >> 4);
-                        mma_ts(tmem + kAccCol, a, bd, idesc_fc1, (first && step == 0) ? 0u : 1u);
-                        if (step == 5) mma_commit(bar(kBarFree + s0));
+                        const uint32_t a =
+                            tmem + kSlotCol0 + (uint32_t)(step < kHalf ? s0 : s1) * kSlotCols + 8u * (step % kHalf);
+                        const uint64_t bd = wdesc + (uint64_t)(((step / kStepsPerBox) * kBoxTx +
+                                                                (step % kStepsPerBox) * 32) >> 4);
+                        if (F8)
+                            mma_ts_f8(tmem + kAccCol, a, bd, idesc_fc1, (first && step == 0) ? 0u : 1u);
+                        else
+                            mma_ts(tmem + kAccCol, a, bd, idesc_fc1, (first && step == 0) ? 0u : 1u);
+                        if (step == kHalf - 1) mma_commit(bar(kBarFree + s0));
                     }
                     if (!ok) break;
                     mma_commit(bar(kBarFree + s1));
@@ -628,19 +681,38 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
             }
             tc_fence_after();
             const uint32_t d = lane_tmem + kSlotCol0 + (uint32_t)s * kSlotCols;
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {  // position x, then x+1: 48 fp32 -> 24 packed words
-                uint32_t f[48];
-                tmem_ld16<0>(d + 48u * h, f);
-                tmem_ld16<16>(d + 48u * h + 16u, f);
-                tmem_ld16<32>(d + 48u * h + 32u, f);
-                tmem_ld_wait();
-                reg_fence(f);
+            if (F8) {  // both positions -> 96 e4m3 bytes = 24 words
                 uint32_t o[24];
 #pragma unroll
-                for (int i = 0; i < 24; ++i) o[i] = relu_pack<FP16>(f[2 * i], f[2 * i + 1]);
-                tmem_st16<0>(d + 24u * h, o);
-                tmem_st8<16>(d + 24u * h + 16u, o);
+                for (int h = 0; h < 2; ++h) {
+                    uint32_t f[48];
+                    tmem_ld16<0>(d + 48u * h, f);
+                    tmem_ld16<16>(d + 48u * h + 16u, f);
+                    tmem_ld16<32>(d + 48u * h + 32u, f);
+                    tmem_ld_wait();
+                    reg_fence(f);
+                    // the conv weights and bias carry kFp8ActScale, so f is already scaled
+#pragma unroll
+                    for (int i = 0; i < 12; ++i)
+                        o[12 * h + i] = relu_e4m3x4(f[4 * i], f[4 * i + 1], f[4 * i + 2], f[4 * i + 3]);
+                }
+                tmem_st16<0>(d, o);
+                tmem_st8<16>(d + 16u, o);
+            } else {
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {  // position x, then x+1: 48 fp32 -> 24 packed words
+                    uint32_t f[48];
+                    tmem_ld16<0>(d + 48u * h, f);
+                    tmem_ld16<16>(d + 48u * h + 16u, f);
+                    tmem_ld16<32>(d + 48u * h + 32u, f);
+                    tmem_ld_wait();
+                    reg_fence(f);
+                    uint32_t o[24];
+#pragma unroll
+                    for (int i = 0; i < 24; ++i) o[i] = relu_pack<FP16>(f[2 * i], f[2 * i + 1]);
+                    tmem_st16<0>(d + 24u * h, o);
+                    tmem_st8<16>(d + 24u * h + 16u, o);
+                }
             }
             tmem_st_wait();
             tc_fence_before();
@@ -714,41 +786,74 @@ float from16(uint16_t u, bool fp16) {
 }  // namespace
 
 cudaError_t init_tc_kernel_attrs() {
-    cudaError_t e = cudaFuncSetAttribute(cnn_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(cnn_tc_kernel<kTcBf16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          kSmemBytesTC);
-    if (e != cudaSuccess) return e;
-    return cudaFuncSetAttribute(cnn_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytesTC);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(cnn_tc_kernel<kTcFp16>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytesTC);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(cnn_tc_kernel<kTcFp8>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytesTC);
+    return e;
 }
 
-cudaError_t prepare_tc_weights(DeviceWeights &w, const emtk_weights &hw, bool fp16) {
-    // dense-1 weights, tiled [K/64][128][64] so that each TMA box is 16 KB of
-    // contiguous memory: tile kb holds W1[kb*64 + kk][nn] at [kb][nn][kk].
-    std::vector<uint16_t> tiles((size_t)kFc1In * kN1);
+double fp8_weight_scale(const float *fc1_w, size_t n) {
+    float m = 0.0f;
+    for (size_t i = 0; i < n; ++i) m = std::fmax(m, std::fabs(fc1_w[i]));
+    if (!(m > 0.0f) || !std::isfinite(m)) return 1.0;
+    // largest 2^k with m * 2^k <= 448, the largest finite e4m3 value
+    int k = 0;
+    while (k < 126 && (double)m * std::ldexp(1.0, k + 1) <= 448.0) ++k;
+    while (k > -126 && (double)m * std::ldexp(1.0, k) > 448.0) --k;
+    return std::ldexp(1.0, k);
+}
+
+cudaError_t prepare_tc_weights(DeviceWeights &w, const emtk_weights &hw, TcMode mode) {
+    const bool fp16 = mode == kTcFp16;
+    const bool f8 = mode == kTcFp8;
+    const size_t nw1 = (size_t)kFc1In * kN1;
+    // dense-1 weights, tiled [K/64][128][64] so that each TMA box is one
+    // contiguous 16 KB (or 8 KB in e4m3): tile kb holds W1[kb*64 + kk][nn] at
+    // [kb][nn][kk].
+    std::vector<uint16_t> tiles(f8 ? 0 : nw1);
+    std::vector<uint8_t> tiles8(f8 ? nw1 : 0);
+    const float sw = f8 ? (float)fp8_weight_scale(hw.fc1_w, nw1) : 1.0f;
     for (int kb = 0; kb < kKBlocks; ++kb)
         for (int nn = 0; nn < kN1; ++nn)
-            for (int kk = 0; kk < kW1Box; ++kk)
-                tiles[((size_t)kb * kN1 + nn) * kW1Box + kk] = to16(hw.fc1_w[(size_t)(kb * kW1Box + kk) * kN1 + nn], fp16);
+            for (int kk = 0; kk < kW1Box; ++kk) {
+                const size_t t = ((size_t)kb * kN1 + nn) * kW1Box + kk;
+                const float v = hw.fc1_w[(size_t)(kb * kW1Box + kk) * kN1 + nn];
+                if (f8)
+                    tiles8[t] = (uint8_t)__nv_cvt_float_to_fp8(v * sw, __NV_SATFINITE, __NV_E4M3);
+                else
+                    tiles[t] = to16(v, fp16);
+            }
+    w.fc1_scale = f8 ? 1.0f / (kFp8ActScale * sw) : 1.0f;
+    w.fc1_w_scale = sw;
     // pair conv B operand [96][32]: row f (< 48) is filter f at x, row 48 + f
     // filter f at x + 1; tap t = 6i + j reads window column j; taps 30 and 31
-    // carry the bias split into a 16-bit head and a 16-bit remainder.
+    // carry the bias split into a 16-bit head and a 16-bit remainder.  In
+    // e4m3 mode weights and bias are multiplied by the activation scale (a
+    // power of two: the rounding to bf16 and the fp32 sums scale exactly).
+    const float cs = f8 ? kFp8ActScale : 1.0f;
     std::vector<uint16_t> cb((size_t)kPairN * kConvK, 0);
     for (int f = 0; f < kF; ++f) {
         for (int i = 0; i < kK; ++i)
             for (int j = 0; j < kK; ++j) {
-                const uint16_t wv = to16(hw.conv_w[(i * kK + j) * kF + f], fp16);
+                const uint16_t wv = to16(hw.conv_w[(i * kK + j) * kF + f] * cs, fp16);
                 cb[(size_t)f * kConvK + 6 * i + j] = wv;              // position x: window columns 0..4
                 cb[(size_t)(kF + f) * kConvK + 6 * i + j + 1] = wv;   // position x+1: window columns 1..5
             }
-        const uint16_t hi = to16(hw.conv_b[f], fp16);
-        const uint16_t lo = to16(hw.conv_b[f] - from16(hi, fp16), fp16);
+        const uint16_t hi = to16(hw.conv_b[f] * cs, fp16);
+        const uint16_t lo = to16(hw.conv_b[f] * cs - from16(hi, fp16), fp16);
         for (int h = 0; h < 2; ++h) {
             cb[(size_t)(h * kF + f) * kConvK + 30] = hi;
             cb[(size_t)(h * kF + f) * kConvK + 31] = lo;
         }
     }
-    cudaError_t e = cudaMalloc(&w.w1_tiles, tiles.size() * 2);
+    const size_t w1_bytes = f8 ? nw1 : nw1 * 2;
+    cudaError_t e = cudaMalloc(&w.w1_tiles, w1_bytes);
     if (e != cudaSuccess) return e;
-    e = cudaMemcpy(w.w1_tiles, tiles.data(), tiles.size() * 2, cudaMemcpyHostToDevice);
+    e = cudaMemcpy(w.w1_tiles, f8 ? (const void *)tiles8.data() : (const void *)tiles.data(), w1_bytes,
+                   cudaMemcpyHostToDevice);
     if (e != cudaSuccess) return e;
     e = cudaMalloc(&w.convB, cb.size() * 2);
     if (e != cudaSuccess) return e;
@@ -762,12 +867,15 @@ cudaError_t prepare_tc_weights(DeviceWeights &w, const emtk_weights &hw, bool fp
     auto encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
     CUtensorMap *map = new CUtensorMap;
     cuuint64_t dims[3] = {(cuuint64_t)kW1Box, (cuuint64_t)kN1, (cuuint64_t)kKBlocks};
-    cuuint64_t strides[2] = {(cuuint64_t)kW1Box * 2, (cuuint64_t)kW1Box * kN1 * 2};
+    const cuuint64_t esz = f8 ? 1 : 2;  // bytes per weight
+    cuuint64_t strides[2] = {(cuuint64_t)kW1Box * esz, (cuuint64_t)kW1Box * kN1 * esz};
     cuuint32_t box[3] = {(cuuint32_t)kW1Box, (cuuint32_t)kN1, 1u};
     cuuint32_t estr[3] = {1u, 1u, 1u};
-    CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_UINT16, 3, w.w1_tiles, dims, strides, box, estr,
-                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    // a box row is 128 bytes (16 bit) or 64 bytes (e4m3): the swizzle span matches it
+    CUresult r = encode(map, f8 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_UINT16, 3, w.w1_tiles,
+                        dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        f8 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) {
         delete map;
         return cudaErrorInvalidValue;
@@ -790,21 +898,28 @@ int streamk_partial_rows(int32_t n, int G) {
     return rows;
 }
 
-cudaError_t launch_cnn_tc(const DeviceWeights &w, const void *src, const HitDesc *desc, bool fp16, int32_t n,
+cudaError_t launch_cnn_tc(const DeviceWeights &w, const void *src, const HitDesc *desc, TcMode mode, int32_t n,
                           int G, float *partials, int n_pad, int *status, int64_t timeout_ns, int debug_stall,
                           cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
     const CUtensorMap &map = *static_cast<const CUtensorMap *>(w.w1_tmap);
     const long long units = (long long)((n + 127) / 128) * kW1Steps;
+    const uint16_t *src16 = static_cast<const uint16_t *>(src);
     dim3 grid(G);
-    if (fp16)
-        cnn_tc_kernel<true><<<grid, kThreadsTC, kSmemBytesTC, s>>>(map, static_cast<const uint16_t *>(src), desc, n,
-                                                                   w.convB, partials, n_pad, units, status,
-                                                                   (long long)timeout_ns, debug_stall);
-    else
-        cnn_tc_kernel<false><<<grid, kThreadsTC, kSmemBytesTC, s>>>(map, static_cast<const uint16_t *>(src), desc, n,
-                                                                    w.convB, partials, n_pad, units, status,
-                                                                    (long long)timeout_ns, debug_stall);
+    switch (mode) {
+    case kTcFp16:
+        cnn_tc_kernel<kTcFp16><<<grid, kThreadsTC, kSmemBytesTC, s>>>(
+            map, src16, desc, n, w.convB, partials, n_pad, units, status, (long long)timeout_ns, debug_stall);
+        break;
+    case kTcFp8:
+        cnn_tc_kernel<kTcFp8><<<grid, kThreadsTC, kSmemBytesTC, s>>>(
+            map, src16, desc, n, w.convB, partials, n_pad, units, status, (long long)timeout_ns, debug_stall);
+        break;
+    default:
+        cnn_tc_kernel<kTcBf16><<<grid, kThreadsTC, kSmemBytesTC, s>>>(
+            map, src16, desc, n, w.convB, partials, n_pad, units, status, (long long)timeout_ns, debug_stall);
+        break;
+    }
     return cudaGetLastError();
 }
 

@@ -100,10 +100,15 @@ struct DeviceWeights {
     float *cls_b = nullptr;
     float *mic_w = nullptr;      // [32]
     float *mic_b = nullptr;
-    uint16_t *w1_tiles = nullptr;  // 16-bit dense-1 weights, tiled for TMA: [1452][128][64]
+    void *w1_tiles = nullptr;      // dense-1 weights, tiled for TMA: [1452][128][64] of 16 bit or e4m3
     uint16_t *convB = nullptr;     // 16-bit conv B operand: [48][32] (taps 0-24, bias hi, bias lo, zeros)
     void *w1_tmap = nullptr;       // host copy of the TMA descriptor (CUtensorMap, 128 B)
+    float fc1_scale = 1.0f;        // dense-1 sums are scaled by this before the bias (EMTK_FP8: 1/(s_a s_w))
+    float fc1_w_scale = 1.0f;      // EMTK_FP8: s_w, the power of two the weights were scaled by
 };
+
+// Operand formats of the tensor-core kernel.
+enum TcMode { kTcBf16 = 0, kTcFp16 = 1, kTcFp8 = 2 };
 
 }  // namespace emtk
 
@@ -159,7 +164,7 @@ cudaError_t launch_cnn_fp32(const DeviceWeights &w, const float *patches, int32_
 // = streamk_partial_rows(n, G).
 // src: 16-bit patches [n][48][48] (desc == nullptr) or the haloed interval
 // images of the hits' planes, located through desc.
-cudaError_t launch_cnn_tc(const DeviceWeights &w, const void *src, const HitDesc *desc, bool fp16, int32_t n,
+cudaError_t launch_cnn_tc(const DeviceWeights &w, const void *src, const HitDesc *desc, TcMode mode, int32_t n,
                           int G, float *partials, int n_pad, int *status, int64_t timeout_ns, int debug_stall,
                           cudaStream_t s);
 int streamk_partial_rows(int32_t n, int G);
@@ -174,7 +179,9 @@ cudaError_t init_fp32_kernel_attrs();
 cudaError_t init_tc_kernel_attrs();
 
 // Host helpers for the tensor-core weights (cnn_tc.cu).
-cudaError_t prepare_tc_weights(DeviceWeights &w, const emtk_weights &hw, bool fp16);
+cudaError_t prepare_tc_weights(DeviceWeights &w, const emtk_weights &hw, TcMode mode);
+// EMTK_FP8 weight scale: the largest power of two s_w with max|W1| s_w <= 448.
+double fp8_weight_scale(const float *fc1_w, size_t n);
 int choose_splits_fp32(int n, int sm_count, int max_splits);
 
 }  // namespace emtk

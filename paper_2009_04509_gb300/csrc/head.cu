@@ -1,5 +1,6 @@
 // Network tail (Sec. 2.2), fp32: sum of the dense-1 partial-sum rows in row
-// order + bias + ReLU, dense 128->32 + ReLU, the 3-way softmax head (track,
+// order, times the dense-1 scale s1 (1, or the inverse of the operand scales
+// of the e4m3 path), + bias + ReLU, dense 128->32 + ReLU, the 3-way softmax head (track,
 // em, none) and the Michel sigmoid head.  One thread per hit: the thread
 // streams its dense-1 outputs four at a time and folds each into the 32
 // dense-2 sums at once (weights broadcast from shared memory), so only the
@@ -14,7 +15,8 @@ constexpr int kThreadsHead = 128;
 constexpr int kManyRows = 4;  // above this many partial rows per hit, reduce them with a warp per hit
 
 __global__ void __launch_bounds__(kThreadsHead) head_kernel(const float *__restrict__ partials, int splits, int G,
-                                                           int n_pad, int32_t n, const float *__restrict__ fc1_b,
+                                                           int n_pad, int32_t n, float s1,
+                                                           const float *__restrict__ fc1_b,
                                                            const float *__restrict__ fc2_w,
                                                            const float *__restrict__ fc2_b,
                                                            const float *__restrict__ cls_w,
@@ -60,8 +62,9 @@ __global__ void __launch_bounds__(kThreadsHead) head_kernel(const float *__restr
             a.w += v.w;
         }
         const float4 bb = *reinterpret_cast<const float4 *>(&b1[4 * c]);
-        const float h1[4] = {fmaxf(a.x + bb.x, 0.f), fmaxf(a.y + bb.y, 0.f), fmaxf(a.z + bb.z, 0.f),
-                             fmaxf(a.w + bb.w, 0.f)};
+        // s1 is a power of two: a * s1 + b rounds once, as a + b does for s1 = 1
+        const float h1[4] = {fmaxf(fmaf(a.x, s1, bb.x), 0.f), fmaxf(fmaf(a.y, s1, bb.y), 0.f),
+                             fmaxf(fmaf(a.z, s1, bb.z), 0.f), fmaxf(fmaf(a.w, s1, bb.w), 0.f)};
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
             const float4 *wr = reinterpret_cast<const float4 *>(&w2[4 * c + e][0]);
@@ -111,7 +114,7 @@ constexpr int kThreadsRows = 256;
 constexpr int kH1Stride = kN1 + 1;  // shared h1 rows padded: thread t reads row t conflict-free
 
 __global__ void __launch_bounds__(kThreadsRows) head_rows_kernel(const float *__restrict__ partials, int splits,
-                                                                int G, int n_pad, int32_t n,
+                                                                int G, int n_pad, int32_t n, float s1,
                                                                 const float *__restrict__ fc1_b,
                                                                 const float *__restrict__ fc2_w,
                                                                 const float *__restrict__ fc2_b,
@@ -154,10 +157,10 @@ __global__ void __launch_bounds__(kThreadsRows) head_rows_kernel(const float *__
             a.w += v.w;
         }
         float *o = h1s + j * kH1Stride + 4 * lane;
-        o[0] = fmaxf(a.x + bb.x, 0.f);
-        o[1] = fmaxf(a.y + bb.y, 0.f);
-        o[2] = fmaxf(a.z + bb.z, 0.f);
-        o[3] = fmaxf(a.w + bb.w, 0.f);
+        o[0] = fmaxf(fmaf(a.x, s1, bb.x), 0.f);
+        o[1] = fmaxf(fmaf(a.y, s1, bb.y), 0.f);
+        o[2] = fmaxf(fmaf(a.z, s1, bb.z), 0.f);
+        o[3] = fmaxf(fmaf(a.w, s1, bb.w), 0.f);
     }
     __syncthreads();
     if (threadIdx.x >= kHitsRows) return;
@@ -214,12 +217,12 @@ cudaError_t launch_head(const DeviceWeights &w, const float *partials, int split
     const int rows = G > 0 ? streamk_partial_rows(n, G) : splits;
     if (rows > kManyRows) {
         head_rows_kernel<<<(n + kHitsRows - 1) / kHitsRows, kThreadsRows, 0, s>>>(
-            partials, splits, G, n_pad, n, w.fc1_b, w.fc2_w, w.fc2_b, w.cls_w, w.cls_b, w.mic_w, w.mic_b, dest,
+            partials, splits, G, n_pad, n, w.fc1_scale, w.fc1_b, w.fc2_w, w.fc2_b, w.cls_w, w.cls_b, w.mic_w, w.mic_b, dest,
             debug_logits);
         return cudaGetLastError();
     }
     head_kernel<<<(n + kThreadsHead - 1) / kThreadsHead, kThreadsHead, 0, s>>>(
-        partials, splits, G, n_pad, n, w.fc1_b, w.fc2_w, w.fc2_b, w.cls_w, w.cls_b, w.mic_w, w.mic_b, dest,
+        partials, splits, G, n_pad, n, w.fc1_scale, w.fc1_b, w.fc2_w, w.fc2_b, w.cls_w, w.cls_b, w.mic_w, w.mic_b, dest,
         debug_logits);
     return cudaGetLastError();
 }

@@ -16,16 +16,16 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libemtk.so")
 
 EMTK_OK, EMTK_ERR_ARG, EMTK_ERR_ALIGN, EMTK_ERR_OOM, EMTK_ERR_CUDA, EMTK_ERR_TIMEOUT, EMTK_ERR_UNSUPPORTED = range(7)
-EMTK_FP32, EMTK_TF32, EMTK_BF16, EMTK_FP16 = 0, 1, 2, 3
+EMTK_FP32, EMTK_TF32, EMTK_BF16, EMTK_FP16, EMTK_FP8 = 0, 1, 2, 3, 4
 EMTK_PATCH_F32, EMTK_PATCH_BF16, EMTK_PATCH_F16 = 0, 1, 2
-PRECISIONS = {"fp32": EMTK_FP32, "tf32": EMTK_TF32, "bf16": EMTK_BF16, "fp16": EMTK_FP16}
+PRECISIONS = {"fp32": EMTK_FP32, "tf32": EMTK_TF32, "bf16": EMTK_BF16, "fp16": EMTK_FP16, "fp8": EMTK_FP8}
 PATCH_FORMATS = {"f32": EMTK_PATCH_F32, "bf16": EMTK_PATCH_BF16, "fp16": EMTK_PATCH_F16}
 KERNELS = ("intervals", "gather", "network", "head", "convert")
 
 EXPORTED = ("emtk_default_options", "emtk_create", "emtk_destroy", "emtk_infer", "emtk_infer_batch",
             "emtk_extract_patches", "emtk_infer_patches", "emtk_check", "emtk_get_stats",
             "emtk_status_string", "emtk_extract_patches_static", "emtk_batcher_create", "emtk_batcher_submit",
-            "emtk_batcher_wait", "emtk_batcher_stats", "emtk_batcher_destroy")
+            "emtk_batcher_wait", "emtk_batcher_stats", "emtk_batcher_destroy", "emtk_get_fp8_scales")
 EMTK_STATIC_SCRATCH_BYTES = 4 << 20
 
 _vp = ctypes.c_void_p
@@ -94,6 +94,8 @@ def load_library(path: str | None = None):
     lib.emtk_batcher_stats.argtypes = [_vp, ctypes.POINTER(ctypes.c_int64), ctypes.POINTER(ctypes.c_int64),
                                        ctypes.POINTER(ctypes.c_int64)]
     lib.emtk_batcher_destroy.argtypes = [_vp]
+    lib.emtk_get_fp8_scales.argtypes = [_vp, _fp, _fp]
+    lib.emtk_get_fp8_scales.restype = ctypes.c_int
     for name in ("emtk_batcher_create", "emtk_batcher_submit", "emtk_batcher_wait", "emtk_batcher_stats",
                  "emtk_batcher_destroy"):
         getattr(lib, name).restype = ctypes.c_int
@@ -229,6 +231,13 @@ def emtk_get_stats(ctx) -> dict:
     _check(load_library().emtk_get_stats(ctx, ctypes.byref(s)), "emtk_get_stats")
     return dict(calls=s.calls, hits=s.hits, launches=s.launches, chunks=s.chunks, batch_hist=list(s.batch_hist),
                 kernel_launches=dict(zip(KERNELS, s.kernel_launches)), kernel_ms=dict(zip(KERNELS, s.kernel_ms)))
+
+
+def emtk_get_fp8_scales(ctx) -> tuple:
+    """(s_a, s_w): the dense-1 operand scales of an "fp8" context, (1, 1) otherwise."""
+    a, w = ctypes.c_float(), ctypes.c_float()
+    _check(load_library().emtk_get_fp8_scales(ctx, ctypes.byref(a), ctypes.byref(w)), "emtk_get_fp8_scales")
+    return float(a.value), float(w.value)
 
 
 # ------------------------------------------------------------------ batcher
