@@ -33,20 +33,20 @@ FLOP_TAIL = 2 * (128 * 32 + 32 * 4)         # 8,448
 FLOP_PER_HIT = FLOP_CONV + FLOP_FC1 + FLOP_TAIL  # 28,444,416
 METRIC = "hit patches/sec on 1 GB300 (extract+CNN); % bf16 tensor peak; gather HBM GB/s"
 
-# DRAM bytes (read + write) of one cnn_tc_kernel launch on the full event, bf16, from
-# one ncu capture of this benchmark (profiles/launch_list_full_event_bf16.md), valid
-# for the kernel source it was taken on: reported as null once that source changes.
-TC_TRAFFIC_BYTES = 50_807_040 + 6_299_904
-TC_TRAFFIC_SOURCE_SHA256 = "16fb956eebfa43b0"
+# DRAM bytes (read + write) of one cnn_tc_kernel launch on the full event, per
+# precision, each from one ncu capture of this benchmark (profiles/launch_list_full_event_*.md),
+# valid for the kernel source they were taken on: reported as null once that source changes.
+TC_TRAFFIC_BYTES = {"bf16": 50_820_608 + 6_388_992, "fp8": 38_856_704 + 1_098_752}
+TC_TRAFFIC_SOURCE_SHA256 = "a8c8335a80c38a4f"
 
 
 def tc_traffic(precision: str, workload: str):
     import hashlib
     src = os.path.join(ROOT, "paper_2009_04509_gb300", "csrc", "cnn_tc.cu")
-    if precision != "bf16" or workload != "full_event" or not os.path.exists(src):
+    if precision not in TC_TRAFFIC_BYTES or workload != "full_event" or not os.path.exists(src):
         return None
     h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
-    return TC_TRAFFIC_BYTES if h == TC_TRAFFIC_SOURCE_SHA256 else None
+    return TC_TRAFFIC_BYTES[precision] if h == TC_TRAFFIC_SOURCE_SHA256 else None
 
 
 def load_peaks():
