@@ -66,6 +66,9 @@ def _bind(path: str):
     lib.or_round_fp16.argtypes = [f32p, f32p, ctypes.c_long]
     lib.or_round_e4m3.argtypes = [f32p, f32p, ctypes.c_long]
     lib.or_set_fp8_scales.argtypes = [ctypes.c_double, ctypes.c_double]
+    lib.or_find_hits.argtypes = [f32p, ctypes.c_int, ctypes.c_int, ctypes.c_long, ctypes.c_float, ctypes.c_long,
+                                 i32p, i32p, i32p, i32p, f32p, f64p]
+    lib.or_find_hits.restype = ctypes.c_long
     lib.or_set_threads.argtypes = [ctypes.c_int]
     lib.or_max_threads.restype = ctypes.c_int
     return lib
@@ -202,6 +205,38 @@ def round_e4m3(x, lib=None):
     x = _c(x, np.float32)
     out = np.zeros(x.shape, np.float32)
     lib.or_round_e4m3(_p(x, ctypes.c_float), _p(out, ctypes.c_float), x.size)
+    return out
+
+
+HIT_FIELDS = ("wire", "tick", "start", "end", "peak", "charge")
+
+
+def find_hits(adc, nticks, threshold, lib=None) -> dict:
+    """Hit finding of Sec. 2.1 as read in the design notes: per wire, each
+    maximal run of ticks with adc > threshold is one hit at the run's largest
+    value (earliest on ties).  ``adc`` [nwires][ld] float32, first ``nticks``
+    columns are data.  Returns a dict of arrays (wire, tick, start, end: int32;
+    peak: float32; charge: float64), ordered by wire then start tick."""
+    lib = lib or load()
+    adc = _c(adc, np.float32)
+    nw, ld = adc.shape
+    args = (_p(adc, ctypes.c_float), nw, int(nticks), ld, ctypes.c_float(threshold))
+
+    def arrays(n):
+        return dict(wire=np.zeros(n, np.int32), tick=np.zeros(n, np.int32), start=np.zeros(n, np.int32),
+                    end=np.zeros(n, np.int32), peak=np.zeros(n, np.float32), charge=np.zeros(n, np.float64))
+
+    def call(a, cap):
+        return lib.or_find_hits(*args, cap, _p(a["wire"], ctypes.c_int32), _p(a["tick"], ctypes.c_int32),
+                                _p(a["start"], ctypes.c_int32), _p(a["end"], ctypes.c_int32),
+                                _p(a["peak"], ctypes.c_float), _p(a["charge"], ctypes.c_double))
+
+    n = call(arrays(1), 0)
+    if n < 0:
+        raise ValueError("or_find_hits: invalid argument")
+    out = arrays(n)
+    if call(out, n) != n:
+        raise RuntimeError("or_find_hits: count changed between calls")
     return out
 
 

@@ -29,6 +29,12 @@
  *   - the conv maps are flattened channels-last: index (y*44 + x)*48 + c;
  *   - softmax outputs are ordered (track, em, none), then the Michel sigmoid.
  *
+ *   Sec. 2.1  Upstream of the patch cut, hits are found on each wire's
+ *             deconvolved waveform (or_find_hits).  The paper does not give
+ *             the algorithm; the reading taken: a hit is a maximal run of
+ *             consecutive ticks whose value exceeds a threshold, placed at
+ *             the run's largest value.
+ *
  * Precision: the patch cut is fp32 by definition (it must be reproduced bit
  * for bit); everything in the network is accumulated in double.  Optional
  * emulating modes round the operands of the two large contractions (patch,
@@ -383,4 +389,59 @@ int or_forward(const or_dims *d, const float *patches, long n,
     free(cb);
     free(w1);
     return fail ? OR_ERR_OOM : OR_OK;
+}
+
+/* ------------------------------------------------------------- hit finding */
+
+/* Hit finding on the deconvolved waveforms (Sec. 2.1), as read in the
+ * design notes.  On each wire w of the plane, a hit is a maximal run of
+ * consecutive ticks t (0 <= t < nticks) with plane[w][t] > threshold
+ * (strictly; a NaN is never above).  For each run:
+ *   start, end  its first and last tick;
+ *   tick        the tick of its largest value, the earliest one on ties;
+ *   peak        that value;
+ *   charge      the sum of its values, accumulated in double.
+ * Hits are listed wire by wire, and within a wire by start tick.  At most
+ * `capacity` hits are written; the return value is the number found (which
+ * may exceed `capacity`), or -1 for an invalid argument. */
+static int above_threshold(float v, float threshold)
+{
+    return v > threshold;
+}
+
+long or_find_hits(const float *plane, int nwires, int nticks, long ld, float threshold, long capacity,
+                  int32_t *wire, int32_t *tick, int32_t *start, int32_t *end, float *peak, double *charge)
+{
+    if (nwires < 0 || nticks < 0 || ld < nticks || capacity < 0 || (nwires > 0 && nticks > 0 && !plane))
+        return -1;
+    long n = 0;
+    for (int w = 0; w < nwires; ++w) {
+        const float *row = plane + (long)w * ld;
+        int t = 0;
+        while (t < nticks) {
+            if (!above_threshold(row[t], threshold)) {
+                ++t;
+                continue;
+            }
+            const int first = t;
+            int best = t;
+            double q = 0.0;
+            while (t < nticks && above_threshold(row[t], threshold)) {
+                if (row[t] > row[best])
+                    best = t;
+                q += (double)row[t];
+                ++t;
+            }
+            if (n < capacity) {
+                wire[n] = w;
+                tick[n] = best;
+                start[n] = first;
+                end[n] = t - 1;
+                peak[n] = row[best];
+                charge[n] = q;
+            }
+            ++n;
+        }
+    }
+    return n;
 }
