@@ -134,7 +134,8 @@ typedef enum {
     EMTK_KERNEL_NETWORK = 2,   /* conv + dense-1 (tensor cores or fp32) */
     EMTK_KERNEL_HEAD = 3,      /* dense-1 sum + dense-2 + heads */
     EMTK_KERNEL_CONVERT = 4,   /* fp32 patches -> 16 bit (emtk_infer_patches) */
-    EMTK_NUM_KERNELS = 5
+    EMTK_KERNEL_HITFIND = 5,   /* hit finding (emtk_find_hits: count, scan, emit) */
+    EMTK_NUM_KERNELS = 6
 } emtk_kernel;
 
 typedef struct {
@@ -217,6 +218,57 @@ EMTK_API emtk_status emtk_check(emtk_ctx *ctx, emtk_stream stream);
 /* Counters since creation.  In profile mode this first waits for the events
  * of every launch not yet read back. */
 EMTK_API emtk_status emtk_get_stats(emtk_ctx *ctx, emtk_stats *out);
+
+/* ---- Hit finding (upstream of the patch cut) ------------------------------
+ *
+ * Sec. 2.1: the hits that the classifier scores are found on the deconvolved
+ * waveform of each wire.  The paper does not give the algorithm; this one
+ * takes the plainest reading.  On each wire, a hit is a maximal run of
+ * consecutive ticks t < nticks whose value is above the threshold
+ * (adc[w][t] > threshold; NaN is never above).  It is placed at the run's
+ * largest value (the earliest tick on ties).  A run is one hit even if it
+ * holds several local maxima (overlapping pulses are not split). */
+
+/* A found hit's run: first and last tick, the value at the peak tick, and
+ * the fp32 sum of the run's values taken in tick order. */
+typedef struct {
+    int32_t start;
+    int32_t end;
+    float peak;
+    float charge;
+} emtk_hit_info;
+
+/* One plane for emtk_find_hits.  d_adc, nwires, nticks and ld are as in
+ * emtk_request (d_adc 16-byte aligned, ld % 4 == 0, ld >= nticks).  Outputs
+ * are ordered by wire, then tick:
+ *   d_hits [capacity]  (wire, peak tick) of each hit: a hit list that
+ *                      emtk_infer / emtk_request take as it is;
+ *   d_info [capacity]  the run of each hit, or NULL;
+ *   n_found            set on return: the number of hits on the plane.  If
+ *                      it exceeds capacity, only the first `capacity` hits
+ *                      are written. */
+typedef struct {
+    const float *d_adc;
+    int32_t nwires;
+    int32_t nticks;
+    int64_t ld;
+    float threshold;
+    int32_t capacity;
+    emtk_hit *d_hits;
+    emtk_hit_info *d_info;
+    int32_t n_found;
+    int32_t reserved;
+} emtk_hitfind_request;
+
+/* Finds the hits of nreq planes (three kernels per group of up to 64
+ * planes: count, scan, emit; the plane is read twice).  Returns once the
+ * results are complete: it synchronises `stream` to fill each n_found.
+ * EMTK_ERR_ARG for negative sizes, ld < nticks, capacity > 0 with a NULL
+ * d_hits, or a plane holding more than 2^31 - 1 possible runs; EMTK_ERR_ALIGN
+ * as for emtk_infer.  The context's workspace serves as scratch, so calls on
+ * one context must not overlap with each other or with its inference calls
+ * on another stream. */
+EMTK_API emtk_status emtk_find_hits(emtk_ctx *ctx, emtk_hitfind_request *reqs, int32_t nreq, emtk_stream stream);
 
 /* The dense-1 operand scales of an EMTK_FP8 context (see emtk_precision):
  * *s_a = 2^-4 and *s_w; 1 and 1 for every other precision.  Either pointer

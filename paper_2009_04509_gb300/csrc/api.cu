@@ -531,6 +531,72 @@ emtk_status emtk_get_stats(emtk_ctx *c, emtk_stats *out) {
     return EMTK_OK;
 }
 
+emtk_status emtk_find_hits(emtk_ctx *c, emtk_hitfind_request *reqs, int32_t nreq, emtk_stream stream) {
+    if (!c || nreq < 0 || (nreq > 0 && !reqs)) return EMTK_ERR_ARG;
+    // the most runs a plane can hold: one per two ticks on every wire
+    auto max_runs = [](const emtk_hitfind_request &q) { return (int64_t)q.nwires * ((q.nticks + 1) / 2); };
+    // scratch (the partial-sum workspace): plane totals in its first 256 bytes, then the
+    // group's per-wire scratch
+    const size_t scratch_bytes = c->ws.partial_elems * sizeof(float) - 256;
+    const int64_t unit_cap = (int64_t)(scratch_bytes / find_hits_scratch_bytes(1));
+    // a plane's units: wire segments of kSegTicks ticks (none without ticks)
+    auto units = [](const emtk_hitfind_request &q) {
+        return q.nticks > 0 ? (int64_t)q.nwires * ((q.nticks + kSegTicks - 1) / kSegTicks) : 0;
+    };
+    for (int32_t i = 0; i < nreq; ++i) {
+        const emtk_hitfind_request &q = reqs[i];
+        if (q.nwires < 0 || q.nticks < 0 || q.ld < q.nticks || q.capacity < 0) return EMTK_ERR_ARG;
+        if (q.capacity > 0 && q.d_hits == nullptr) return EMTK_ERR_ARG;
+        if (q.nwires > 0 && q.nticks > 0 && q.d_adc == nullptr) return EMTK_ERR_ARG;
+        if (max_runs(q) > INT32_MAX || units(q) > unit_cap) return EMTK_ERR_ARG;
+        if (q.d_adc != nullptr && (!aligned16(q.d_adc) || (q.ld % 4) != 0)) return EMTK_ERR_ALIGN;
+        if ((reinterpret_cast<uintptr_t>(q.d_hits) & 7u) != 0 || (reinterpret_cast<uintptr_t>(q.d_info) & 3u) != 0)
+            return EMTK_ERR_ALIGN;
+    }
+    for (int32_t i = 0; i < nreq; ++i) reqs[i].n_found = 0;
+    if (nreq == 0) return EMTK_OK;
+    DeviceGuard g(c->device);
+    if (!g.ok) return EMTK_ERR_CUDA;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    int32_t *totals = reinterpret_cast<int32_t *>(c->ws.partials);
+    void *scratch = reinterpret_cast<char *>(c->ws.partials) + 256;
+    int32_t i = 0;
+    while (i < nreq) {
+        // a group: up to kMaxHfPlanes planes whose units fit the scratch
+        HfTable t{};
+        int64_t U = 0;
+        const int32_t first = i;
+        while (i < nreq && t.n < kMaxHfPlanes) {
+            const emtk_hitfind_request &q = reqs[i];
+            const int64_t nu = units(q);
+            if (t.n > 0 && U + nu > unit_cap) break;
+            HfDesc &d = t.r[t.n++];
+            d.adc = q.d_adc;
+            d.hits = q.d_hits;
+            d.info = q.d_info;
+            d.ld = q.ld;
+            d.unit0 = U;
+            d.nticks = q.nticks;
+            d.nseg = (q.nticks + kSegTicks - 1) / kSegTicks;
+            d.capacity = q.capacity;
+            d.thr = q.threshold;
+            U += nu;
+            ++i;
+        }
+        cudaError_t e;
+        {
+            Prof prof(c, EMTK_KERNEL_HITFIND, s);
+            e = launch_find_hits(t, U, scratch, totals, s);
+        }
+        int32_t h_tot[kMaxHfPlanes];
+        if (e == cudaSuccess) e = cudaMemcpyAsync(h_tot, totals, sizeof(int32_t) * t.n, cudaMemcpyDeviceToHost, s);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+        if (e != cudaSuccess) return cuda_status(e);
+        for (int r = 0; r < t.n; ++r) reqs[first + r].n_found = h_tot[r];
+    }
+    return EMTK_OK;
+}
+
 emtk_status emtk_get_fp8_scales(const emtk_ctx *c, float *s_a, float *s_w) {
     if (!c) return EMTK_ERR_ARG;
     const bool f8 = c->opt.precision == EMTK_FP8;

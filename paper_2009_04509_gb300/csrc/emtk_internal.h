@@ -77,6 +77,28 @@ struct ReqTable {
     ReqDesc r[kMaxReqPerLaunch];
 };
 
+// Planes of one hit-finding launch group (emtk_find_hits).  The unit of work
+// is a wire segment of kSegTicks ticks; a plane has nwires * nseg units, and
+// unit0 is its first unit in the group's concatenated unit list.
+constexpr int kMaxHfPlanes = 64;
+constexpr int kSegTicks = 2048;
+struct HfDesc {
+    const float *adc;
+    emtk_hit *hits;
+    emtk_hit_info *info;
+    int64_t ld;
+    int64_t unit0;
+    int32_t nticks;
+    int32_t nseg;
+    int32_t capacity;
+    float thr;
+};
+struct HfTable {
+    int32_t n;
+    int32_t pad;
+    HfDesc r[kMaxHfPlanes];
+};
+
 // Per-context workspace (device).
 struct Workspace {
     void *dimg = nullptr;        // interval images of the planes of one launch
@@ -156,6 +178,11 @@ cudaError_t launch_convert_patches(const float *src, void *dst, emtk_patch_forma
 cudaError_t launch_hit_desc(const ReqTable &t, int64_t g0, int32_t count, HitDesc *desc, float **dest,
                             int out_stride, cudaStream_t s);
 cudaError_t launch_fill_dest(float *scores, int out_stride, float **dest, int32_t n, cudaStream_t s);
+// Hit finding of the group's planes (hitfind.cu): scratch holds
+// find_hits_scratch_bytes(U) bytes (16-byte aligned) for the group's U
+// units; totals[r] receives plane r's hit count.
+size_t find_hits_scratch_bytes(int64_t nunits);
+cudaError_t launch_find_hits(const HfTable &t, int64_t nunits, void *scratch, int32_t *totals, cudaStream_t s);
 
 // Network: dense-1 partial sums [splits][n_pad][128] from patches.
 cudaError_t launch_cnn_fp32(const DeviceWeights &w, const float *patches, int32_t n, int splits,

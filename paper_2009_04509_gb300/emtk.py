@@ -20,12 +20,13 @@ EMTK_FP32, EMTK_TF32, EMTK_BF16, EMTK_FP16, EMTK_FP8 = 0, 1, 2, 3, 4
 EMTK_PATCH_F32, EMTK_PATCH_BF16, EMTK_PATCH_F16 = 0, 1, 2
 PRECISIONS = {"fp32": EMTK_FP32, "tf32": EMTK_TF32, "bf16": EMTK_BF16, "fp16": EMTK_FP16, "fp8": EMTK_FP8}
 PATCH_FORMATS = {"f32": EMTK_PATCH_F32, "bf16": EMTK_PATCH_BF16, "fp16": EMTK_PATCH_F16}
-KERNELS = ("intervals", "gather", "network", "head", "convert")
+KERNELS = ("intervals", "gather", "network", "head", "convert", "hitfind")
 
 EXPORTED = ("emtk_default_options", "emtk_create", "emtk_destroy", "emtk_infer", "emtk_infer_batch",
             "emtk_extract_patches", "emtk_infer_patches", "emtk_check", "emtk_get_stats",
             "emtk_status_string", "emtk_extract_patches_static", "emtk_batcher_create", "emtk_batcher_submit",
-            "emtk_batcher_wait", "emtk_batcher_stats", "emtk_batcher_destroy", "emtk_get_fp8_scales")
+            "emtk_batcher_wait", "emtk_batcher_stats", "emtk_batcher_destroy", "emtk_get_fp8_scales",
+            "emtk_find_hits")
 EMTK_STATIC_SCRATCH_BYTES = 4 << 20
 
 _vp = ctypes.c_void_p
@@ -50,7 +51,13 @@ class emtk_request(ctypes.Structure):
 class emtk_stats(ctypes.Structure):
     _fields_ = [("calls", ctypes.c_uint64), ("hits", ctypes.c_uint64), ("launches", ctypes.c_uint64),
                 ("chunks", ctypes.c_uint64), ("batch_hist", ctypes.c_uint64 * 8),
-                ("kernel_launches", ctypes.c_uint64 * 5), ("kernel_ms", ctypes.c_double * 5)]
+                ("kernel_launches", ctypes.c_uint64 * 6), ("kernel_ms", ctypes.c_double * 6)]
+
+
+class emtk_hitfind_request(ctypes.Structure):
+    _fields_ = [("d_adc", _vp), ("nwires", ctypes.c_int32), ("nticks", ctypes.c_int32), ("ld", ctypes.c_int64),
+                ("threshold", ctypes.c_float), ("capacity", ctypes.c_int32), ("d_hits", _vp), ("d_info", _vp),
+                ("n_found", ctypes.c_int32), ("reserved", ctypes.c_int32)]
 
 
 class EmtkError(RuntimeError):
@@ -96,6 +103,8 @@ def load_library(path: str | None = None):
     lib.emtk_batcher_destroy.argtypes = [_vp]
     lib.emtk_get_fp8_scales.argtypes = [_vp, _fp, _fp]
     lib.emtk_get_fp8_scales.restype = ctypes.c_int
+    lib.emtk_find_hits.argtypes = [_vp, ctypes.POINTER(emtk_hitfind_request), ctypes.c_int32, _vp]
+    lib.emtk_find_hits.restype = ctypes.c_int
     for name in ("emtk_batcher_create", "emtk_batcher_submit", "emtk_batcher_wait", "emtk_batcher_stats",
                  "emtk_batcher_destroy"):
         getattr(lib, name).restype = ctypes.c_int
@@ -231,6 +240,27 @@ def emtk_get_stats(ctx) -> dict:
     _check(load_library().emtk_get_stats(ctx, ctypes.byref(s)), "emtk_get_stats")
     return dict(calls=s.calls, hits=s.hits, launches=s.launches, chunks=s.chunks, batch_hist=list(s.batch_hist),
                 kernel_launches=dict(zip(KERNELS, s.kernel_launches)), kernel_ms=dict(zip(KERNELS, s.kernel_ms)))
+
+
+def emtk_find_hits(ctx, planes, stream=None) -> list:
+    """Hit finding (see include/emtk.h) on several planes in one call.
+    ``planes``: list of (adc [nwires][ld] float32 device tensor, nticks, threshold,
+    hits [capacity][2] int32 device tensor, info [capacity][4] int32 device tensor
+    or None).  info columns: start, end, then peak and charge as float32 bits
+    (``info[:, 2:].view(torch.float32)``).  Returns the number of hits found per
+    plane (which may exceed a plane's capacity); the call synchronises the stream."""
+    reqs = (emtk_hitfind_request * max(1, len(planes)))()
+    for i, (adc, nticks, thr, hits, info) in enumerate(planes):
+        q = reqs[i]
+        q.d_adc = _ptr(adc)
+        q.nwires, q.ld = adc.shape
+        q.nticks = int(nticks)
+        q.threshold = float(thr)
+        q.capacity = hits.shape[0]
+        q.d_hits = _ptr(hits)
+        q.d_info = _ptr(info) if info is not None else None
+    _check(load_library().emtk_find_hits(ctx, reqs, len(planes), _stream(stream)), "emtk_find_hits")
+    return [int(reqs[i].n_found) for i in range(len(planes))]
 
 
 def emtk_get_fp8_scales(ctx) -> tuple:

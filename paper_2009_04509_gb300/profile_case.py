@@ -3,10 +3,13 @@ with ncu.
 
     python -m paper_2009_04509_gb300.profile_case --mode event   # one APA, 20,000 hits
     python -m paper_2009_04509_gb300.profile_case --mode patches --hits 30000
+    python -m paper_2009_04509_gb300.profile_case --mode hitfind          # full event, threshold 15
 
 `event` runs one APA (6 planes, 800/800/480 wires x 6000 ticks, 20,000 hits)
 through emtk_infer_batch, the call the benchmark times on a full event;
-`patches` runs N pre-cut patches through emtk_infer_patches.  The path runs
+`patches` runs N pre-cut patches through emtk_infer_patches; `hitfind` runs
+emtk_find_hits on the 18 planes of the full event (368.6 MB of samples) and
+checks the hit counts against a first run.  The path runs
 twice (capture the second launch with `ncu -s 1 -c 1`), and the context's
 status word is checked, so that a run that ends with exit code 0 was a
 correct, complete one.  Inputs are synthetic and seeded; the device holds a
@@ -25,7 +28,7 @@ from paper_2009_04509_gb300 import emtk, synth  # noqa: E402
 
 def main() -> int:
     ap = argparse.ArgumentParser()
-    ap.add_argument("--mode", default="event", choices=["event", "patches"])
+    ap.add_argument("--mode", default="event", choices=["event", "patches", "hitfind"])
     ap.add_argument("--hits", type=int, default=30000, help="patches mode: number of patches")
     ap.add_argument("--precision", default="bf16", choices=["bf16", "fp16", "fp8", "fp32"])
     ap.add_argument("--runs", type=int, default=2)
@@ -34,6 +37,21 @@ def main() -> int:
     import torch
     dev = torch.device("cuda:0")
     w = synth.he_normal_weights(0)
+    if args.mode == "hitfind":
+        planes = synth.full_event(seed=0)
+        ctx = emtk.emtk_create(w, precision="bf16")
+        cap = 262_144
+        items = [(torch.from_numpy(p.adc).to(dev), p.nticks, 15.0, torch.empty((cap, 2), dtype=torch.int32, device=dev),
+                  torch.empty((cap, 4), dtype=torch.int32, device=dev)) for p in planes]
+        try:
+            counts = [emtk.emtk_find_hits(ctx, items) for _ in range(args.runs)]
+        finally:
+            emtk.emtk_destroy(ctx)
+        if any(c != counts[0] for c in counts):
+            print("hit counts differ between runs", file=sys.stderr)
+            return 1
+        print(f"ok: hitfind, {sum(counts[0])} hits on {len(planes)} planes, {args.runs} runs")
+        return 0
     if args.mode == "event":
         planes = synth.apa(seed=0)
         ctx = emtk.emtk_create(w, precision=args.precision)

@@ -60,13 +60,34 @@ def test_default_options(lib):
     assert o.wait_timeout_ns == 2_000_000_000 and o.debug_stall == 0 and o.profile == 0
 
 
-def test_struct_layouts_match_header(lib):
-    # emtk_request: ptr, 2 x int32, int64, ptr, int32 (+pad), ptr
-    assert ctypes.sizeof(emtk.emtk_request) == 48
-    assert emtk.emtk_request.d_scores.offset == 40
-    assert ctypes.sizeof(emtk.emtk_options) == 32
-    assert ctypes.sizeof(emtk.emtk_weights) == 80
-    assert ctypes.sizeof(emtk.emtk_stats) == 176
+ABI_STRUCTS = ("emtk_request", "emtk_options", "emtk_weights", "emtk_stats", "emtk_hitfind_request")
+
+
+def test_struct_layouts_match_header(lib, tmp_path):
+    """Every struct the binding mirrors has the header's size and field
+    offsets, as a C compiler lays them out."""
+    import shutil
+    import subprocess
+    if shutil.which("gcc") is None:
+        pytest.skip("gcc not available")
+    inc = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
+    lines = ["#include <stddef.h>", "#include <stdio.h>", '#include "emtk.h"', "int main(void) {"]
+    for name in ABI_STRUCTS:
+        lines.append(f'printf("{name} %zu\\n", sizeof({name}));')
+        for f, _ in getattr(emtk, name)._fields_:
+            lines.append(f'printf("{name}.{f} %zu\\n", offsetof({name}, {f}));')
+    lines.append("return 0; }")
+    src = tmp_path / "layout.c"
+    src.write_text("\n".join(lines))
+    exe = tmp_path / "layout"
+    subprocess.run(["gcc", "-I", inc, str(src), "-o", str(exe)], check=True)
+    want = dict(l.split() for l in subprocess.run([str(exe)], capture_output=True, text=True,
+                                                   check=True).stdout.splitlines())
+    for name in ABI_STRUCTS:
+        st = getattr(emtk, name)
+        assert ctypes.sizeof(st) == int(want[name]), name
+        for f, _ in st._fields_:
+            assert getattr(st, f).offset == int(want[f"{name}.{f}"]), f"{name}.{f}"
 
 
 def test_argument_errors_without_device(lib):
@@ -78,6 +99,7 @@ def test_argument_errors_without_device(lib):
     assert lib.emtk_check(null, None) == emtk.EMTK_ERR_ARG
     assert lib.emtk_get_stats(null, None) == emtk.EMTK_ERR_ARG
     assert lib.emtk_destroy(null) == emtk.EMTK_OK
+    assert lib.emtk_find_hits(null, None, 0, None) == emtk.EMTK_ERR_ARG
     out = ctypes.c_void_p()
     assert lib.emtk_create(None, None, 0, ctypes.byref(out)) == emtk.EMTK_ERR_ARG and not out.value
     w = synth.he_normal_weights(0, dims=dict(P=6, R=3, F=2, N1=2, N2=2, NC=3))
