@@ -532,6 +532,19 @@ def run_sweep(args, rank, world, local_rank):
 
 
 HITFIND_THRESHOLD = 15.0  # 5 sigma of the synthetic planes' noise
+# DRAM bytes (read + write) of one hf_find_kernel launch on the full event, from one ncu
+# capture of this workload (profiles/hitfind_full_event.md); null once hitfind.cu changes.
+HF_TRAFFIC_BYTES = 369_571_584 + 6_144_000
+HF_TRAFFIC_SOURCE_SHA256 = "99117707123cde30"
+
+
+def hf_traffic():
+    import hashlib
+    src = os.path.join(ROOT, "paper_2009_04509_gb300", "csrc", "hitfind.cu")
+    if not os.path.exists(src):
+        return None
+    h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    return HF_TRAFFIC_BYTES if h == HF_TRAFFIC_SOURCE_SHA256 else None
 
 
 def run_hitfind(args, rank, world, local_rank):
@@ -592,8 +605,22 @@ def run_hitfind(args, rank, world, local_rank):
                         "achieved": alg_bytes / (kern_ms / 1e3) / 1e9, "peak": peaks["hbm"], "unit": "GB/s",
                         "frac": alg_bytes / (kern_ms / 1e3) / 1e9 / peaks["hbm"],
                         "peak_source": f"{peaks['source']} HBM copy", "algorithmic_bytes": alg_bytes,
-                        "launch_ms": kern_ms, "traffic": None},
+                        "launch_ms": kern_ms, "traffic": hf_traffic(), "traffic_kernel": "hf_find_kernel",
+                        "traffic_unit": "bytes per launch (ncu dram__bytes_read.sum + dram__bytes_write.sum)"},
            "clocks": clk}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        oracle.build()
+        lib = oracle.load()
+        t0 = time.perf_counter()
+        reps = 0
+        while time.perf_counter() - t0 < 2.0:  # whole steps, at least 2 s
+            n_cpu = sum(oracle.find_hits(p.adc, p.nticks, HITFIND_THRESHOLD, lib=lib)["wire"].size for p in planes)
+            reps += 1
+        t_cpu = (time.perf_counter() - t0) / reps
+        out["cpu_baseline"] = {"value": samples / t_cpu, "unit": "samples/s", "cores": 1, "kind": "oracle",
+                               "sample": f"whole steps: or_find_hits on all 18 planes, {reps} times "
+                                         f"({t_cpu:.3f} s each, {n_cpu} hits), one thread"}
     if rank == 0:
         print(json.dumps(out))
 
