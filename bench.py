@@ -36,8 +36,8 @@ METRIC = "hit patches/sec on 1 GB300 (extract+CNN); % bf16 tensor peak; gather H
 # DRAM bytes (read + write) of one cnn_tc_kernel launch on the full event, per
 # precision, each from one ncu capture of this benchmark (profiles/launch_list_full_event_*.md),
 # valid for the kernel source they were taken on: reported as null once that source changes.
-TC_TRAFFIC_BYTES = {"bf16": 50_820_608 + 6_388_992, "fp8": 38_856_704 + 1_098_752}
-TC_TRAFFIC_SOURCE_SHA256 = "a8c8335a80c38a4f"
+TC_TRAFFIC_BYTES = {"bf16": 50_805_504 + 6_386_432, "fp8": 38_858_496 + 1_097_216}
+TC_TRAFFIC_SOURCE_SHA256 = "36b0a0db98821ace"
 
 
 def tc_traffic(precision: str, workload: str):
