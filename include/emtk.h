@@ -174,6 +174,25 @@ EMTK_API emtk_status emtk_infer(emtk_ctx *ctx, const float *d_adc, int32_t nwire
  * batching (Sec. 3.2).  Requests with nhits == 0 are allowed. */
 EMTK_API emtk_status emtk_infer_batch(emtk_ctx *ctx, const emtk_request *reqs, int32_t nreq, emtk_stream stream);
 
+/* emtk_infer_batch with HOST buffers: each request's d_adc, d_hits and
+ * d_scores point to host memory (the same layouts; pinned memory lets the
+ * copies overlap).  The planes and hit lists are copied to one of two device
+ * staging areas of the context on its own copy stream, the batch runs on
+ * `stream`, and the scores are copied back on `stream`; the call returns
+ * once all of it is enqueued.  Consecutive calls use the two areas in turn,
+ * so the copy-in of call i+1 overlaps the kernels of call i (the inference
+ * server's input transfer, Sec. 3.3, hidden behind the previous batch).
+ *   - The host buffers must stay valid and unchanged until `stream` has
+ *     completed the call (cudaStreamSynchronize, or an event recorded on
+ *     `stream` after the call), and the scores are final only then.
+ *   - A staging area grows to the largest call it has served (a cudaMalloc,
+ *     after waiting for that area's previous call).
+ *   - ld % 4 == 0 and ld >= nticks, as for emtk_infer_batch; no alignment is
+ *     required of the host pointers.
+ * Errors as for emtk_infer_batch; EMTK_ERR_OOM if a staging area cannot grow. */
+EMTK_API emtk_status emtk_infer_batch_host(emtk_ctx *ctx, const emtk_request *reqs, int32_t nreq,
+                                           emtk_stream stream);
+
 /* Patch cut only (Sec. 2.1): d_patches [nhits][48][48] of `fmt`.  F32 is the
  * exact fp32 value; BF16 / F16 are that value rounded to nearest-even. */
 EMTK_API emtk_status emtk_extract_patches(emtk_ctx *ctx, const float *d_adc, int32_t nwires, int32_t nticks,

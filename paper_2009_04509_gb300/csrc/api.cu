@@ -73,6 +73,16 @@ void free_ctx(emtk_ctx *c) {
     for (void *p : {c->ws.dimg, c->ws.patches, (void *)c->ws.dest, (void *)c->ws.partials, (void *)c->ws.status,
                     (void *)c->ws.hdesc})
         if (p) cudaFree(p);
+    if (c->copy_stream) {
+        cudaStreamSynchronize(c->copy_stream);
+        cudaStreamDestroy(c->copy_stream);
+    }
+    for (auto &st : c->stage) {
+        if (st.compute_done) cudaEventSynchronize(st.compute_done);
+        if (st.buf) cudaFree(st.buf);
+        if (st.copy_done) cudaEventDestroy(st.copy_done);
+        if (st.compute_done) cudaEventDestroy(st.compute_done);
+    }
     delete c;
 }
 
@@ -529,6 +539,86 @@ emtk_status emtk_get_stats(emtk_ctx *c, emtk_stats *out) {
     }
     *out = c->stats;
     return EMTK_OK;
+}
+
+emtk_status emtk_infer_batch_host(emtk_ctx *c, const emtk_request *reqs, int32_t nreq, emtk_stream stream) {
+    if (!c || nreq < 0 || (nreq > 0 && !reqs)) return EMTK_ERR_ARG;
+    // staging layout: each plane at a 256-byte boundary, then the hit lists, then the scores
+    const int stride = out_stride(c);
+    auto up = [](size_t x) { return (x + 255) & ~(size_t)255; };
+    std::vector<size_t> off_adc(nreq), off_hits(nreq), off_sc(nreq);
+    size_t need = 0;
+    for (int32_t i = 0; i < nreq; ++i) {
+        const emtk_request &q = reqs[i];
+        if (q.nwires < 0 || q.nticks < 0 || q.nhits < 0 || q.ld < q.nticks || (q.ld % 4) != 0) return EMTK_ERR_ARG;
+        if (q.nhits > 0 && (!q.d_adc || !q.d_hits || !q.d_scores)) return EMTK_ERR_ARG;
+        off_adc[i] = need;
+        need = up(need + (q.nhits > 0 ? (size_t)q.nwires * (size_t)q.ld * sizeof(float) : 0));
+    }
+    for (int32_t i = 0; i < nreq; ++i) {
+        off_hits[i] = need;
+        need = up(need + (size_t)reqs[i].nhits * sizeof(emtk_hit));
+    }
+    for (int32_t i = 0; i < nreq; ++i) {
+        off_sc[i] = need;
+        need = up(need + (size_t)reqs[i].nhits * stride * sizeof(float));
+    }
+    if (need == 0) return EMTK_OK;
+    DeviceGuard g(c->device);
+    if (!g.ok) return EMTK_ERR_CUDA;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaSuccess;
+    if (!c->copy_stream) e = cudaStreamCreateWithFlags(&c->copy_stream, cudaStreamNonBlocking);
+    emtk_ctx::HostStage &st = c->stage[c->host_calls % 2];
+    if (e == cudaSuccess && !st.copy_done) e = cudaEventCreateWithFlags(&st.copy_done, cudaEventDisableTiming);
+    if (e == cudaSuccess && !st.compute_done) e = cudaEventCreateWithFlags(&st.compute_done, cudaEventDisableTiming);
+    if (e == cudaSuccess && st.bytes < need) {  // grow: wait for the area's last call, then reallocate
+        if (st.used) e = cudaEventSynchronize(st.compute_done);
+        if (e == cudaSuccess && st.buf) e = cudaFree(st.buf);
+        st.buf = nullptr;
+        st.bytes = 0;
+        if (e == cudaSuccess) e = cudaMalloc(&st.buf, need);
+        if (e == cudaSuccess) st.bytes = need;
+    }
+    if (e != cudaSuccess) return cuda_status(e);
+    char *base = static_cast<char *>(st.buf);
+    // copy in on the copy stream, once the area's previous call is done with it
+    if (st.used) e = cudaStreamWaitEvent(c->copy_stream, st.compute_done, 0);
+    std::vector<emtk_request> dq(reqs, reqs + nreq);
+    for (int32_t i = 0; i < nreq && e == cudaSuccess; ++i) {
+        const emtk_request &q = reqs[i];
+        if (q.nhits == 0) {  // nothing of it is read: no host pointer reaches the batch
+            dq[i].d_adc = nullptr;
+            dq[i].d_hits = nullptr;
+            dq[i].d_scores = nullptr;
+            continue;
+        }
+        e = cudaMemcpyAsync(base + off_adc[i], q.d_adc, (size_t)q.nwires * q.ld * sizeof(float),
+                            cudaMemcpyHostToDevice, c->copy_stream);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(base + off_hits[i], q.d_hits, (size_t)q.nhits * sizeof(emtk_hit),
+                                cudaMemcpyHostToDevice, c->copy_stream);
+        dq[i].d_adc = reinterpret_cast<const float *>(base + off_adc[i]);
+        dq[i].d_hits = reinterpret_cast<const emtk_hit *>(base + off_hits[i]);
+        dq[i].d_scores = reinterpret_cast<float *>(base + off_sc[i]);
+    }
+    if (e == cudaSuccess) e = cudaEventRecord(st.copy_done, c->copy_stream);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(s, st.copy_done, 0);
+    if (e != cudaSuccess) return cuda_status(e);
+    // the batch on the caller's stream, then the scores back to the caller's buffers
+    emtk_status r = emtk_infer_batch(c, dq.data(), nreq, stream);
+    for (int32_t i = 0; i < nreq && r == EMTK_OK; ++i) {
+        const emtk_request &q = reqs[i];
+        if (q.nhits == 0) continue;
+        e = cudaMemcpyAsync(q.d_scores, base + off_sc[i], (size_t)q.nhits * stride * sizeof(float),
+                            cudaMemcpyDeviceToHost, s);
+        if (e != cudaSuccess) r = cuda_status(e);
+    }
+    e = cudaEventRecord(st.compute_done, s);
+    if (e != cudaSuccess && r == EMTK_OK) r = cuda_status(e);
+    st.used = true;
+    c->host_calls++;
+    return r;
 }
 
 emtk_status emtk_find_hits(emtk_ctx *c, emtk_hitfind_request *reqs, int32_t nreq, emtk_stream stream) {

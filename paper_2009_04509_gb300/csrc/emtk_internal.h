@@ -150,6 +150,17 @@ struct emtk_ctx {
     emtk::Workspace ws;
     emtk_stats stats{};
     bool owns_weights = true;  // false for a batcher lane, which shares its parent's weights
+    // emtk_infer_batch_host: two device staging areas used alternately, filled on
+    // the context's copy stream; compute_done[k] marks the end of the last call
+    // that used area k (its scores copied out), copy_done[k] the end of its copy.
+    struct HostStage {
+        void *buf = nullptr;
+        size_t bytes = 0;
+        cudaEvent_t copy_done = nullptr, compute_done = nullptr;
+        bool used = false;
+    } stage[2];
+    cudaStream_t copy_stream = nullptr;
+    uint64_t host_calls = 0;
 };
 
 namespace emtk {

@@ -26,7 +26,7 @@ EXPORTED = ("emtk_default_options", "emtk_create", "emtk_destroy", "emtk_infer",
             "emtk_extract_patches", "emtk_infer_patches", "emtk_check", "emtk_get_stats",
             "emtk_status_string", "emtk_extract_patches_static", "emtk_batcher_create", "emtk_batcher_submit",
             "emtk_batcher_wait", "emtk_batcher_stats", "emtk_batcher_destroy", "emtk_get_fp8_scales",
-            "emtk_find_hits")
+            "emtk_find_hits", "emtk_infer_batch_host")
 EMTK_STATIC_SCRATCH_BYTES = 4 << 20
 
 _vp = ctypes.c_void_p
@@ -104,6 +104,8 @@ def load_library(path: str | None = None):
     lib.emtk_get_fp8_scales.argtypes = [_vp, _fp, _fp]
     lib.emtk_get_fp8_scales.restype = ctypes.c_int
     lib.emtk_find_hits.argtypes = [_vp, ctypes.POINTER(emtk_hitfind_request), ctypes.c_int32, _vp]
+    lib.emtk_infer_batch_host.argtypes = [_vp, ctypes.POINTER(emtk_request), ctypes.c_int32, _vp]
+    lib.emtk_infer_batch_host.restype = ctypes.c_int
     lib.emtk_find_hits.restype = ctypes.c_int
     for name in ("emtk_batcher_create", "emtk_batcher_submit", "emtk_batcher_wait", "emtk_batcher_stats",
                  "emtk_batcher_destroy"):
@@ -206,6 +208,15 @@ def emtk_infer_batch(ctx, items, stream=None) -> None:
     items = list(items)
     reqs = make_requests(items)
     _check(load_library().emtk_infer_batch(ctx, reqs, len(items), _stream(stream)), "emtk_infer_batch")
+
+
+def emtk_infer_batch_host(ctx, items, stream=None) -> None:
+    """emtk_infer_batch with host (CPU) tensors: (adc, nticks, hits, scores) per
+    request.  Returns once the work is enqueued; the scores are final when the
+    stream has completed, and the tensors must stay alive until then."""
+    items = list(items)
+    reqs = make_requests(items)
+    _check(load_library().emtk_infer_batch_host(ctx, reqs, len(items), _stream(stream)), "emtk_infer_batch_host")
 
 
 def emtk_extract_patches(ctx, adc, nticks: int, hits, patches, fmt: str = "f32", stream=None) -> None:

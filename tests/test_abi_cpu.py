@@ -100,6 +100,7 @@ def test_argument_errors_without_device(lib):
     assert lib.emtk_get_stats(null, None) == emtk.EMTK_ERR_ARG
     assert lib.emtk_destroy(null) == emtk.EMTK_OK
     assert lib.emtk_find_hits(null, None, 0, None) == emtk.EMTK_ERR_ARG
+    assert lib.emtk_infer_batch_host(null, None, 0, None) == emtk.EMTK_ERR_ARG
     out = ctypes.c_void_p()
     assert lib.emtk_create(None, None, 0, ctypes.byref(out)) == emtk.EMTK_ERR_ARG and not out.value
     w = synth.he_normal_weights(0, dims=dict(P=6, R=3, F=2, N1=2, N2=2, NC=3))
