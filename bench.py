@@ -176,8 +176,30 @@ def cpu_oracle_rate(planes, weights, budget_s: float = 15.0):
         t_net += time.perf_counter() - t1
         done += sel.size
     per_hit = t_cut / nh + t_net / done
+    # the same network on one thread, on a few hits
+    oracle.set_threads(1, lib=lib)
+    n1 = min(8, allp.shape[0])
+    t1 = time.perf_counter()
+    oracle.forward(allp[idx[:n1]], weights, lib=lib)
+    t_one = (time.perf_counter() - t1) / n1
+    oracle.set_threads(threads, lib=lib)
+    single = 1.0 / (t_cut / nh + t_one)
     return 1.0 / per_hit, threads, (f"patch cut of all {nh} hits ({t_cut:.2f} s) + network (fp64) on "
-                                    f"{done} random hits ({t_net:.2f} s), {threads} OpenMP threads")
+                                    f"{done} random hits ({t_net:.2f} s), {threads} OpenMP threads"), single
+
+
+def reduce_over_ranks(local_ms: float, local_units: int, dist, device):
+    """Replicas (one independent event per rank, no exchange in the data
+    path): the job's time is the slowest rank's, its work the sum of the
+    ranks' units.  Returns (max ms, total units); single process: the inputs."""
+    if not dist:
+        return local_ms, local_units
+    import torch
+    t = torch.tensor([local_ms], dtype=torch.float64, device=device)
+    u = torch.tensor([float(local_units)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(u, op=dist.ReduceOp.SUM)
+    return float(t.item()), int(round(u.item()))
 
 
 # -------------------------------------------------------------------- main
@@ -270,13 +292,9 @@ def main():
     assert rc == emtk.EMTK_OK, emtk.status_string(rc)
     st = emtk.emtk_get_stats(ctx)
     step_ms = [a.elapsed_time(b) for a, b in ev]
-    total_ms = float(sum(step_ms))
-    if dist:
-        t = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms, all_hits = reduce_over_ranks(float(sum(step_ms)), nhits * args.steps, dist, dev)
     ms_per_step = total_ms / args.steps
-    value = world * nhits * args.steps / (total_ms / 1e3)
+    value = all_hits / (total_ms / 1e3)
 
     kms = {k: st["kernel_ms"][k] - base["kernel_ms"][k] for k in emtk.KERNELS}
     kn = {k: st["kernel_launches"][k] - base["kernel_launches"][k] for k in emtk.KERNELS}
@@ -334,6 +352,8 @@ def main():
                        "kernels": "interval_image_kernel + " + ("gather_kernel" if args.precision == "fp32"
                                                                else "hit_desc_kernel"),
                        "ms_per_step": cut_ms},
+        "step_ms_stats": {"median": statistics.median(step_ms), "min": min(step_ms), "max": max(step_ms),
+                          "mean": total_ms / args.steps, "n": len(step_ms)},
         "kernel_ms_per_step": {k: v / args.steps for k, v in kms.items()},
         "whole_step_frac_of_bf16_peak": value * FLOP_PER_HIT / 1e12 / peaks["bf16"] / world,
         "clocks": clk,
@@ -341,8 +361,9 @@ def main():
     if e2e:
         out["e2e"] = e2e
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        rate, cores, sample = cpu_oracle_rate(planes, weights, args.cpu_budget)
-        out["cpu_baseline"] = {"value": rate, "unit": "hits/s", "cores": cores, "kind": "oracle", "sample": sample}
+        rate, cores, sample, single = cpu_oracle_rate(planes, weights, args.cpu_budget)
+        out["cpu_baseline"] = {"value": rate, "unit": "hits/s", "cores": cores, "kind": "oracle", "sample": sample,
+                               "value_single_thread": single}
     emtk.emtk_destroy(ctx)
     if rank == 0:
         print(json.dumps(out))
@@ -630,20 +651,22 @@ def run_reference(args, rank, world):
     planes = synth.full_event(seed=0) if args.workload == "full_event" else synth.apa(seed=0)
     weights = synth.he_normal_weights(0)
     budget = max(1.0, min(args.cpu_budget, 120.0 / max(1, args.steps + args.warmup)))
-    rates = []
+    rates, singles = [], []
     sample = ""
     cores = 0
     for i in range(args.warmup + args.steps):
-        rate, cores, sample = cpu_oracle_rate(planes, weights, budget)
+        rate, cores, sample, single = cpu_oracle_rate(planes, weights, budget)
         if i >= args.warmup:
             rates.append(rate)
+            singles.append(single)
     value = float(statistics.median(rates))
     nh = sum(p.nhits for p in planes)
     out = {"impl": "reference", "metric": METRIC, "value": value, "unit": "hits/s", "n_gpus": world,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": nh / value * 1e3, "higher_is_better": True,
            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
            "config": {"workload": "full 6-APA event: 18 planes x 6000 ticks, 60,000 hits (CPU oracle, sampled)"},
-           "cpu_baseline": {"value": value, "unit": "hits/s", "cores": cores, "kind": "oracle", "sample": sample},
+           "cpu_baseline": {"value": value, "unit": "hits/s", "cores": cores, "kind": "oracle", "sample": sample,
+                            "value_single_thread": float(statistics.median(singles))},
            "e2e": {"value": value, "unit": "hits/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(out))
 
