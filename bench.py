@@ -188,6 +188,21 @@ def cpu_oracle_rate(planes, weights, budget_s: float = 15.0):
                                     f"{done} random hits ({t_net:.2f} s), {threads} OpenMP threads"), single
 
 
+WORKLOADS = {
+    "full_event": "full 6-APA event: 18 planes (800/800/960 wires) x 6000 ticks, 60,000 hits, one emtk_infer_batch",
+    "apa": "one APA: planes 800/800/480 x 6000 ticks, 20,000 hits, one emtk_infer per plane",
+    "single": "one collection plane: 480 wires x 6000 ticks, 256 hits on 5 tracks, one emtk_infer",
+}
+
+
+def workload_planes(workload: str, seed: int):
+    if workload == "full_event":
+        return synth.full_event(seed=seed)
+    if workload == "apa":
+        return synth.apa(seed=seed)
+    return [synth.single_plane(seed=seed)]
+
+
 def reduce_over_ranks(local_ms: float, local_units: int, dist, device):
     """Replicas (one independent event per rank, no exchange in the data
     path): the job's time is the slowest rank's, its work the sum of the
@@ -209,7 +224,7 @@ def main():
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="emtk", choices=["emtk", "reference"])
-    ap.add_argument("--workload", default="full_event", choices=["full_event", "apa", "service", "sweep", "hitfind"])
+    ap.add_argument("--workload", default="full_event", choices=["full_event", "apa", "single", "service", "sweep", "hitfind"])
     ap.add_argument("--clients", type=int, default=64, help="service workload: client threads (one event each)")
     ap.add_argument("--streams", type=int, default=8, help="service workload: batcher streams")
     ap.add_argument("--max-delay-us", type=int, default=500, help="service workload: batcher delay")
@@ -240,7 +255,7 @@ def main():
         dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
 
     from paper_2009_04509_gb300 import emtk
-    planes = synth.full_event(seed=rank) if args.workload == "full_event" else synth.apa(seed=rank)
+    planes = workload_planes(args.workload, rank)
     weights = synth.he_normal_weights(0)
     nhits = sum(p.nhits for p in planes)
     dev = torch.device("cuda", local_rank)
@@ -331,11 +346,10 @@ def main():
         "vs_baseline": None,
         "dtype": args.precision,
         "data": "synthetic (seeded ProtoDUNE-SP-shaped planes and hits; He-normal seed-0 weights)",
-        "config": {"workload": ("full 6-APA event: 18 planes (800/800/960 wires) x 6000 ticks, 60,000 hits, "
-                                "one emtk_infer_batch") if args.workload == "full_event" else
-                   "one APA: planes 800/800/480 x 6000 ticks, 20,000 hits, one emtk_infer per plane",
+        "config": {"workload": WORKLOADS[args.workload],
                    "hits_per_step": nhits, "planes": len(planes), "precision": args.precision,
-                   "l2": "flushed between steps (256 MiB write); planes (368.6 MB) exceed L2",
+                   "l2": "flushed between steps (256 MiB write)" + ("; planes (368.6 MB) exceed L2"
+                                                                    if args.workload == "full_event" else ""),
                    "parallelism": f"replicas x{world} (independent events, no collective)"},
         "gpu_launches": launches,
         "roofline": {"bound": "tensor", "kernel": "cnn_tc_kernel (conv 5x5x48 + dense-1, tcgen05)"
@@ -648,7 +662,7 @@ def run_reference(args, rank, world):
     bounded sample of it."""
     if rank != 0:
         return
-    planes = synth.full_event(seed=0) if args.workload == "full_event" else synth.apa(seed=0)
+    planes = workload_planes(args.workload, 0)
     weights = synth.he_normal_weights(0)
     budget = max(1.0, min(args.cpu_budget, 120.0 / max(1, args.steps + args.warmup)))
     rates, singles = [], []
@@ -664,7 +678,7 @@ def run_reference(args, rank, world):
     out = {"impl": "reference", "metric": METRIC, "value": value, "unit": "hits/s", "n_gpus": world,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": nh / value * 1e3, "higher_is_better": True,
            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-           "config": {"workload": "full 6-APA event: 18 planes x 6000 ticks, 60,000 hits (CPU oracle, sampled)"},
+           "config": {"workload": WORKLOADS.get(args.workload, args.workload) + " (CPU oracle, sampled)"},
            "cpu_baseline": {"value": value, "unit": "hits/s", "cores": cores, "kind": "oracle", "sample": sample,
                             "value_single_thread": float(statistics.median(singles))},
            "e2e": {"value": value, "unit": "hits/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
