@@ -108,11 +108,14 @@ __global__ void __launch_bounds__(kThreadsHead) head_kernel(const float *__restr
 // tiles are split over many CTAs): one warp per hit sums the rows, lane l
 // taking dense-1 outputs 4l .. 4l+3 of every row (512 contiguous bytes per
 // row), and writes bias + ReLU to shared memory; then one thread per hit
-// finishes as above.  32 hits per block.
-constexpr int kHitsRows = 32;
+// finishes as above.  HITS hits per block: 8 for small launches (more
+// blocks, so more rows summed at once), 32 above kSmallLaunch hits (fewer
+// blocks loading the dense-2 weights).
 constexpr int kThreadsRows = 256;
+constexpr int kSmallLaunch = 2048;
 constexpr int kH1Stride = kN1 + 1;  // shared h1 rows padded: thread t reads row t conflict-free
 
+template <int kHitsRows>
 __global__ void __launch_bounds__(kThreadsRows) head_rows_kernel(const float *__restrict__ partials, int splits,
                                                                 int G, int n_pad, int32_t n, float s1,
                                                                 const float *__restrict__ fc1_b,
@@ -216,9 +219,14 @@ cudaError_t launch_head(const DeviceWeights &w, const float *partials, int split
     // most partial rows a hit has: many when a small launch spreads each tile over many CTAs
     const int rows = G > 0 ? streamk_partial_rows(n, G) : splits;
     if (rows > kManyRows) {
-        head_rows_kernel<<<(n + kHitsRows - 1) / kHitsRows, kThreadsRows, 0, s>>>(
-            partials, splits, G, n_pad, n, w.fc1_scale, w.fc1_b, w.fc2_w, w.fc2_b, w.cls_w, w.cls_b, w.mic_w, w.mic_b, dest,
-            debug_logits);
+        if (n <= kSmallLaunch)
+            head_rows_kernel<8><<<(n + 7) / 8, kThreadsRows, 0, s>>>(
+                partials, splits, G, n_pad, n, w.fc1_scale, w.fc1_b, w.fc2_w, w.fc2_b, w.cls_w, w.cls_b, w.mic_w,
+                w.mic_b, dest, debug_logits);
+        else
+            head_rows_kernel<32><<<(n + 31) / 32, kThreadsRows, 0, s>>>(
+                partials, splits, G, n_pad, n, w.fc1_scale, w.fc1_b, w.fc2_w, w.fc2_b, w.cls_w, w.cls_b, w.mic_w,
+                w.mic_b, dest, debug_logits);
         return cudaGetLastError();
     }
     head_kernel<<<(n + kThreadsHead - 1) / kThreadsHead, kThreadsHead, 0, s>>>(
