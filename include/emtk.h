@@ -280,8 +280,9 @@ typedef struct {
 } emtk_hitfind_request;
 
 /* Finds the hits of nreq planes (three kernels per group of up to 64
- * planes: count, scan, emit; the plane is read twice).  Returns once the
- * results are complete: it synchronises `stream` to fill each n_found.
+ * planes: find, per-plane scan, place; each sample is read once).  Returns
+ * once the results are complete: it synchronises `stream` to fill each
+ * n_found.
  * EMTK_ERR_ARG for negative sizes, ld < nticks, capacity > 0 with a NULL
  * d_hits, or a plane holding more than 2^31 - 1 possible runs; EMTK_ERR_ALIGN
  * as for emtk_infer.  The context's workspace serves as scratch, so calls on
