@@ -9,8 +9,9 @@
  * ReLU, a 3-way softmax (track, em, none) and a 1-way sigmoid (Michel).
  *
  * Conventions for every entry point below:
- *   - Pointers named d_* are device memory owned by the caller.  They must
- *     stay valid until the work enqueued on the caller's stream completes.
+ *   - Pointers named d_* are device memory owned by the caller (host memory
+ *     in emtk_infer_batch_host, which says so).  They must stay valid until
+ *     the work enqueued on the caller's stream completes.
  *   - All work is enqueued on the caller's stream; nothing synchronises
  *     unless stated.  A context may be used from one stream at a time.
  *   - Argument errors are reported synchronously and enqueue nothing.
@@ -134,7 +135,7 @@ typedef enum {
     EMTK_KERNEL_NETWORK = 2,   /* conv + dense-1 (tensor cores or fp32) */
     EMTK_KERNEL_HEAD = 3,      /* dense-1 sum + dense-2 + heads */
     EMTK_KERNEL_CONVERT = 4,   /* fp32 patches -> 16 bit (emtk_infer_patches) */
-    EMTK_KERNEL_HITFIND = 5,   /* hit finding (emtk_find_hits: count, scan, emit) */
+    EMTK_KERNEL_HITFIND = 5,   /* hit finding (emtk_find_hits: find, scan, place) */
     EMTK_NUM_KERNELS = 6
 } emtk_kernel;
 
