@@ -1,117 +1,151 @@
 // fp32 network path on CUDA cores (EMTK_FP32): conv 5x5x48 + ReLU fused
-// with dense-1 (Sec. 2.2), split over the dense-1 input dimension.
+// with dense-1 (Sec. 2.2), split over the dense-1 input dimension (the conv
+// positions) into `splits` segments.
 //
-// Block = 32 hits x one segment of conv positions.  Per position the block
-// computes the 32 x 48 conv activations into shared memory from a 5-row
-// band of the 32 patches, stages the 48 x 128 dense-1 rows of that position
-// and accumulates 2 hits x 8 outputs per thread in fp32.  Segment partial
-// sums go to partials[segment][hit][128]; the head kernel adds them in
-// segment order, so results are deterministic.
+// Block = 128 hits x one segment of conv positions, 256 threads.  Per
+// position the block
+//   - computes the 128 x 48 conv activations (thread: one hit, 24 filters)
+//     from a 5-row band of the hits' patches held in shared memory (rows
+//     kept by row % 5, one new row per output row), transposed into act[48][128];
+//   - multiplies them into the dense-1 sums with the position's 48 x 128
+//     weights, which cp.async brought into one of two shared buffers while
+//     the previous position was computed: thread (hit group g, output group
+//     o) accumulates hits 8g..8g+7 x outputs 8o..8o+7 in 64 registers, 16
+//     FMAs per shared-memory load.
+// Segment partial sums go to partials[segment][hit][128]; the head kernel
+// adds them in segment order, so results are deterministic.
 #include "emtk_internal.h"
 
 namespace emtk {
 namespace {
 
-constexpr int kHT = 32;      // hits per block
+constexpr int kHT = 128;      // hits per block
 constexpr int kThreads = 256;
-constexpr int kSmemBytes = (kF * kN1 + kK * kHT * kPatch + kHT * (kF + 1) + kK * kK * kF + kF) * 4;
+constexpr int kBandStride = kPatch + 1;  // 49: conflict-free per-hit reads
+constexpr int kW1Pos = kF * kN1;         // 6144 weights of one position (24 KB)
+// shared memory: band[5][128][49], w1[2][48][128], act[48][128], cw[25][48], cb[48]
+constexpr int kSmemFloats = kK * kHT * kBandStride + 2 * kW1Pos + kF * kHT + kK * kK * kF + kF;
+constexpr int kSmemBytes = kSmemFloats * 4;
+static_assert(kSmemBytes <= 232448, "shared memory budget");
 
-__global__ void __launch_bounds__(kThreads) cnn_fp32_kernel(const float *__restrict__ patches, int n,
-                                                            const float *__restrict__ conv_w,
-                                                            const float *__restrict__ conv_b,
-                                                            const float *__restrict__ fc1_w, int splits,
-                                                            float *__restrict__ partials, int n_pad) {
+__device__ __forceinline__ void cp_async16(float *smem_dst, const float *gmem_src) {
+    const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(smem_dst));
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d), "l"(gmem_src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_prev() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
+
+// The 48 x 128 dense-1 weights of position p into dst (each thread 6 x 16 bytes).
+__device__ __forceinline__ void load_w1(float *dst, const float *__restrict__ fc1_w, int p, int tid) {
+    const float *src = fc1_w + (int64_t)p * kW1Pos;
+#pragma unroll
+    for (int k = 0; k < kW1Pos / 4 / kThreads; ++k) {
+        const int i = (tid + k * kThreads) * 4;
+        cp_async16(dst + i, src + i);
+    }
+}
+
+// Patch row `prow` of the block's 128 hits into band slot prow % 5 (zero past n).
+__device__ __forceinline__ void load_band_row(float *band, const float *__restrict__ patches, int n, int hit0, int prow,
+                                              int tid) {
+    float *slot = band + (prow % kK) * kHT * kBandStride;
+    for (int i = tid; i < kHT * kPatch / 4; i += kThreads) {
+        const int h = i / (kPatch / 4), c4 = i - h * (kPatch / 4);
+        const int gh = hit0 + h;
+        float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (gh < n) v = __ldg(reinterpret_cast<const float4 *>(patches + (int64_t)gh * kPatchElems + prow * kPatch) + c4);
+        float *d = slot + h * kBandStride + 4 * c4;
+        d[0] = v.x;
+        d[1] = v.y;
+        d[2] = v.z;
+        d[3] = v.w;
+    }
+}
+
+__global__ void __launch_bounds__(kThreads, 1) cnn_fp32_kernel(const float *__restrict__ patches, int n,
+                                                               const float *__restrict__ conv_w,
+                                                               const float *__restrict__ conv_b,
+                                                               const float *__restrict__ fc1_w, int splits,
+                                                               float *__restrict__ partials, int n_pad) {
     extern __shared__ float4 smem_f4[];
-    auto &w1s = *reinterpret_cast<float (*)[kF][kN1]>(smem_f4);
-    auto &band = *reinterpret_cast<float (*)[kK][kHT][kPatch]>(&w1s[kF][0]);  // rows by (row % 5)
-    auto &act = *reinterpret_cast<float (*)[kHT][kF + 1]>(&band[kK][0][0]);
-    auto &cw = *reinterpret_cast<float (*)[kK * kK][kF]>(&act[kHT][0]);
-    float *cb = &cw[kK * kK][0];
+    float *band = reinterpret_cast<float *>(smem_f4);  // [5][128][49]
+    float *w1 = band + kK * kHT * kBandStride;          // [2][48][128]
+    float *act = w1 + 2 * kW1Pos;                       // [48][128]
+    float *cw = act + kF * kHT;                         // [25][48]
+    float *cb = cw + kK * kK * kF;                      // [48]
 
     const int tid = threadIdx.x;
     const int hit0 = blockIdx.x * kHT;
     const int seg = blockIdx.y;
     const int p_begin = (int)((int64_t)seg * kPos / splits);
     const int p_end = (int)((int64_t)(seg + 1) * kPos / splits);
-
-    for (int i = tid; i < kK * kK * kF; i += kThreads) cw[i / kF][i % kF] = conv_w[i];
+    for (int i = tid; i < kK * kK * kF; i += kThreads) cw[i] = conv_w[i];
     for (int i = tid; i < kF; i += kThreads) cb[i] = conv_b[i];
 
-    // dense-1 mapping: hits 2*hp, 2*hp+1; outputs n0..n0+7
-    const int hp = tid >> 4;
-    const int n0 = (tid & 15) * 8;
-    float acc[2][8];
+    const int g = tid >> 4, o = tid & 15;        // dense-1: hits 8g.., outputs 8o..
+    const int ch = tid >> 1, f0 = (tid & 1) * 24;  // conv: hit ch, filters f0..f0+23
+    float acc[8][8];
 #pragma unroll
-    for (int a = 0; a < 2; ++a)
+    for (int i = 0; i < 8; ++i)
 #pragma unroll
-        for (int e = 0; e < 8; ++e) acc[a][e] = 0.0f;
+        for (int j = 0; j < 8; ++j) acc[i][j] = 0.0f;
 
-    // conv mapping: hit ch = tid >> 3, filters c0..c0+5
-    const int ch = tid >> 3;
-    const int c0 = (tid & 7) * 6;
-
-    int band_y = -100;  // first patch row held in band
+    if (p_begin < p_end) load_w1(w1, fc1_w, p_begin, tid);
+    cp_async_commit();
+    int band_y = -1;
     for (int p = p_begin; p < p_end; ++p) {
-        const int y = p / kQ;
-        const int x = p - y * kQ;
-        if (y != band_y) {
-            __syncthreads();
-            for (int i = tid; i < kK * kHT * kPatch; i += kThreads) {
-                const int rr = i / (kHT * kPatch);
-                const int rem = i - rr * kHT * kPatch;
-                const int h = rem / kPatch;
-                const int col = rem - h * kPatch;
-                const int prow = y + rr;
-                const int gh = hit0 + h;
-                band[prow % kK][h][col] = gh < n ? patches[(int64_t)gh * kPatchElems + prow * kPatch + col] : 0.0f;
-            }
+        const int y = p / kQ, x = p - y * kQ;
+        // the next position's weights into the other buffer (free since the last barrier)
+        if (p + 1 < p_end) load_w1(w1 + ((p + 1 - p_begin) & 1) * kW1Pos, fc1_w, p + 1, tid);
+        cp_async_commit();
+        if (y != band_y) {  // rows y..y+4: all five at the segment's start, then the one new row
+            for (int r = band_y < 0 ? y : y + kK - 1; r < y + kK; ++r) load_band_row(band, patches, n, hit0, r, tid);
             band_y = y;
+            __syncthreads();
         }
-        // stage the 48 x 128 dense-1 rows of this position
-        const float4 *src = reinterpret_cast<const float4 *>(fc1_w + (int64_t)p * kF * kN1);
-        for (int i = tid; i < kF * kN1 / 4; i += kThreads)
-            reinterpret_cast<float4 *>(&w1s[0][0])[i] = __ldg(src + i);
-        __syncthreads();
-        // conv + ReLU for (hit ch, filters c0..c0+5)
-        float s[6];
+        // conv + ReLU of hit ch, filters f0 .. f0+23, transposed into act
+        float s[24];
 #pragma unroll
-        for (int f = 0; f < 6; ++f) s[f] = cb[c0 + f];
+        for (int f = 0; f < 24; ++f) s[f] = cb[f0 + f];
 #pragma unroll
         for (int i = 0; i < kK; ++i) {
-            const float *row = &band[(y + i) % kK][ch][x];
+            const float *row = band + ((y + i) % kK) * kHT * kBandStride + ch * kBandStride + x;
 #pragma unroll
             for (int j = 0; j < kK; ++j) {
                 const float v = row[j];
+                const float *wrow = cw + (i * kK + j) * kF + f0;
 #pragma unroll
-                for (int f = 0; f < 6; ++f) s[f] = fmaf(v, cw[i * kK + j][c0 + f], s[f]);
+                for (int f = 0; f < 24; ++f) s[f] = fmaf(v, wrow[f], s[f]);
             }
         }
 #pragma unroll
-        for (int f = 0; f < 6; ++f) act[ch][c0 + f] = fmaxf(s[f], 0.0f);
+        for (int f = 0; f < 24; ++f) act[(f0 + f) * kHT + ch] = fmaxf(s[f], 0.0f);
+        cp_async_wait_prev();  // this position's weights have landed
         __syncthreads();
-        // dense-1 accumulate
+        // dense-1: 8 hits x 8 outputs per thread
+        const float *wp = w1 + ((p - p_begin) & 1) * kW1Pos;
 #pragma unroll 4
         for (int c = 0; c < kF; ++c) {
-            const float a0 = act[2 * hp][c];
-            const float a1 = act[2 * hp + 1][c];
-            const float4 wa = *reinterpret_cast<const float4 *>(&w1s[c][n0]);
-            const float4 wb = *reinterpret_cast<const float4 *>(&w1s[c][n0 + 4]);
-            const float w[8] = {wa.x, wa.y, wa.z, wa.w, wb.x, wb.y, wb.z, wb.w};
+            const float4 a0 = *reinterpret_cast<const float4 *>(act + c * kHT + 8 * g);
+            const float4 a1 = *reinterpret_cast<const float4 *>(act + c * kHT + 8 * g + 4);
+            const float4 b0 = *reinterpret_cast<const float4 *>(wp + c * kN1 + 8 * o);
+            const float4 b1 = *reinterpret_cast<const float4 *>(wp + c * kN1 + 8 * o + 4);
+            const float a[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+            const float b[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
 #pragma unroll
-            for (int e = 0; e < 8; ++e) {
-                acc[0][e] = fmaf(a0, w[e], acc[0][e]);
-                acc[1][e] = fmaf(a1, w[e], acc[1][e]);
-            }
+            for (int i = 0; i < 8; ++i)
+#pragma unroll
+                for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
         }
         __syncthreads();
     }
 #pragma unroll
-    for (int a = 0; a < 2; ++a) {
-        const int gh = hit0 + 2 * hp + a;
+    for (int i = 0; i < 8; ++i) {
+        const int gh = hit0 + 8 * g + i;
         if (gh < n) {
-            float *dst = partials + ((int64_t)seg * n_pad + gh) * kN1 + n0;
-            reinterpret_cast<float4 *>(dst)[0] = make_float4(acc[a][0], acc[a][1], acc[a][2], acc[a][3]);
-            reinterpret_cast<float4 *>(dst)[1] = make_float4(acc[a][4], acc[a][5], acc[a][6], acc[a][7]);
+            float *dst = partials + ((int64_t)seg * n_pad + gh) * kN1 + 8 * o;
+            reinterpret_cast<float4 *>(dst)[0] = make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
+            reinterpret_cast<float4 *>(dst)[1] = make_float4(acc[i][4], acc[i][5], acc[i][6], acc[i][7]);
         }
     }
 }
@@ -122,9 +156,10 @@ cudaError_t init_fp32_kernel_attrs() {
     return cudaFuncSetAttribute(cnn_fp32_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
 }
 
+// K splits: about four waves of one-block-per-SM work, at least 16 positions per split.
 int choose_splits_fp32(int n, int sm_count, int max_splits) {
     const int blocks = (n + kHT - 1) / kHT;
-    int s = (2 * sm_count + blocks - 1) / blocks;
+    int s = (4 * sm_count + blocks - 1) / blocks;
     if (s > kPos / 16) s = kPos / 16;
     if (s > max_splits) s = max_splits;
     return s < 1 ? 1 : s;
