@@ -58,12 +58,22 @@ def load_peaks():
     return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, source="fallback")
 
 
+# The fp32 path runs on the CUDA cores: one FMA (2 FLOP) per lane per clock,
+# 128 fp32 lanes per SM (4 sub-partitions x 32), 152 SMs, 2070 MHz maximum SM clock.
+FP32_ALU_TFLOPS = 152 * 128 * 2 * 2070e6 / 1e12
+FP32_ALU_SOURCE = "derived: 152 SMs x 128 fp32 lanes x 2 FLOP (FMA) x 2070 MHz"
+
+
 def network_peak(precision: str, peaks: dict):
-    """Tensor peak (TFLOP/s, sustained) of the network kernel's own mix of
-    operand types: the 16-bit paths run at the bf16 rate; the fp8 path runs
-    the conv at the bf16 rate and dense-1 on e4m3 operands at twice it (the
-    nominal fp8 : bf16 ratio), so its peak is the FLOP-weighted harmonic mix."""
+    """Peak of the network kernel (TFLOP/s).  The fp32 path is CUDA-core
+    arithmetic, against the derived fp32 FMA rate.  Otherwise the sustained
+    tensor peak of the network kernel's own mix of operand types: the 16-bit
+    paths run at the bf16 rate; the fp8 path runs the conv at the bf16 rate
+    and dense-1 on e4m3 operands at twice it (the nominal fp8 : bf16 ratio),
+    so its peak is the FLOP-weighted harmonic mix."""
     p = peaks["bf16_sus"]
+    if precision == "fp32":
+        return FP32_ALU_TFLOPS, FP32_ALU_SOURCE
     if precision != "fp8":
         return p, f"{peaks['source']} bf16 sustained"
     return ((FLOP_CONV + FLOP_FC1) / (FLOP_CONV / p + FLOP_FC1 / (2.0 * p)),
@@ -352,11 +362,12 @@ def main():
                                                                     if args.workload == "full_event" else ""),
                    "parallelism": f"replicas x{world} (independent events, no collective)"},
         "gpu_launches": launches,
-        "roofline": {"bound": "tensor", "kernel": "cnn_tc_kernel (conv 5x5x48 + dense-1, tcgen05)"
+        "roofline": {"bound": "alu" if args.precision == "fp32" else "tensor", "kernel": "cnn_tc_kernel (conv 5x5x48 + dense-1, tcgen05)"
                      if args.precision != "fp32" else "cnn_fp32_kernel",
                      "achieved": achieved, "peak": net_peak, "unit": "TFLOP/s",
                      "frac": achieved / net_peak,
-                     "peak_source": net_peak_src, "frac_of_burst": achieved / net_peak * peaks["bf16_sus"] / peaks["bf16"],
+                     "peak_source": net_peak_src, "frac_of_burst": None if args.precision == "fp32"
+                     else achieved / net_peak * peaks["bf16_sus"] / peaks["bf16"],
                      "flop_per_hit": FLOP_CONV + FLOP_FC1, "hits_per_launch": hits_per_launch,
                      "launch_ms": net_ms, "traffic": tc_traffic(args.precision, args.workload),
                      "traffic_unit": "bytes per launch (ncu dram__bytes_read.sum + dram__bytes_write.sum)"},
@@ -633,7 +644,7 @@ def run_hitfind(args, rank, world, local_rank):
                       "samples_per_step": samples, "hits_found": nfound,
                       "l2": "flushed between steps (256 MiB write); planes (368.6 MB) exceed L2"},
            "hits_per_s": nfound / (step_ms / 1e3),
-           "roofline": {"bound": "hbm", "kernel": "hf_count_kernel + hf_scan_kernel + hf_emit_kernel",
+           "roofline": {"bound": "hbm", "kernel": "hf_find_kernel + hf_scan_kernel + hf_place_kernel",
                         "achieved": alg_bytes / (kern_ms / 1e3) / 1e9, "peak": peaks["hbm"], "unit": "GB/s",
                         "frac": alg_bytes / (kern_ms / 1e3) / 1e9 / peaks["hbm"],
                         "peak_source": f"{peaks['source']} HBM copy", "algorithmic_bytes": alg_bytes,

@@ -135,7 +135,7 @@ typedef enum {
     EMTK_KERNEL_NETWORK = 2,   /* conv + dense-1 (tensor cores or fp32) */
     EMTK_KERNEL_HEAD = 3,      /* dense-1 sum + dense-2 + heads */
     EMTK_KERNEL_CONVERT = 4,   /* fp32 patches -> 16 bit (emtk_infer_patches) */
-    EMTK_KERNEL_HITFIND = 5,   /* hit finding (emtk_find_hits: find, scan, place) */
+    EMTK_KERNEL_HITFIND = 5,   /* hit finding (emtk_find_hits: chunk-sum memset, find, place) */
     EMTK_NUM_KERNELS = 6
 } emtk_kernel;
 
@@ -250,7 +250,11 @@ EMTK_API emtk_status emtk_get_stats(emtk_ctx *ctx, emtk_stats *out);
  * holds several local maxima (overlapping pulses are not split). */
 
 /* A found hit's run: first and last tick, the value at the peak tick, and
- * the fp32 sum of the run's values taken in tick order. */
+ * the fp32 sum of the run's values.  The summation order is fixed (the same
+ * result on every call): a run within one aligned group of 4 ticks sums in
+ * tick order, a longer run adds a pairwise sum per 32-tick step from its
+ * start, steps in order; the error stays within the usual fp32 bound of a
+ * sum of that length. */
 typedef struct {
     int32_t start;
     int32_t end;
@@ -280,8 +284,9 @@ typedef struct {
     int32_t reserved;
 } emtk_hitfind_request;
 
-/* Finds the hits of nreq planes (three kernels per group of up to 64
- * planes: find, per-plane scan, place; each sample is read once).  Returns
+/* Finds the hits of nreq planes (per group of up to 64 planes: a memset of
+ * the chunk sums, then two kernels, find and place; each sample is read
+ * once, units with more than 128 runs per 2048 ticks twice).  Returns
  * once the results are complete: it synchronises `stream` to fill each
  * n_found.
  * EMTK_ERR_ARG for negative sizes, ld < nticks, capacity > 0 with a NULL

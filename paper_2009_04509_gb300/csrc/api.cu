@@ -628,7 +628,7 @@ emtk_status emtk_find_hits(emtk_ctx *c, emtk_hitfind_request *reqs, int32_t nreq
     // scratch (the partial-sum workspace): plane totals in its first 256 bytes, then the
     // group's per-wire scratch
     const size_t scratch_bytes = c->ws.partial_elems * sizeof(float) - 256;
-    const int64_t unit_cap = (int64_t)(scratch_bytes / find_hits_scratch_bytes(1));
+    const int64_t unit_cap = find_hits_unit_cap(scratch_bytes);
     // a plane's units: wire segments of kSegTicks ticks (none without ticks)
     auto units = [](const emtk_hitfind_request &q) {
         return q.nticks > 0 ? (int64_t)q.nwires * ((q.nticks + kSegTicks - 1) / kSegTicks) : 0;

@@ -88,6 +88,7 @@ struct HfDesc {
     emtk_hit_info *info;
     int64_t ld;
     int64_t unit0;
+    int64_t chunk0;  // the plane's first chunk of units (set by launch_find_hits)
     int32_t nticks;
     int32_t nseg;
     int32_t capacity;
@@ -189,10 +190,11 @@ cudaError_t launch_convert_patches(const float *src, void *dst, emtk_patch_forma
 cudaError_t launch_hit_desc(const ReqTable &t, int64_t g0, int32_t count, HitDesc *desc, float **dest,
                             int out_stride, cudaStream_t s);
 cudaError_t launch_fill_dest(float *scores, int out_stride, float **dest, int32_t n, cudaStream_t s);
-// Hit finding of the group's planes (hitfind.cu): scratch holds
-// find_hits_scratch_bytes(U) bytes (16-byte aligned) for the group's U
-// units; totals[r] receives plane r's hit count.
-size_t find_hits_scratch_bytes(int64_t nunits);
+// Hit finding of the group's planes (hitfind.cu): scratch (256-byte aligned)
+// holds the launch's chunk sums and per-unit run slots; find_hits_unit_cap
+// gives the most units that scratch_bytes holds.  totals[r] receives plane
+// r's hit count.
+int64_t find_hits_unit_cap(size_t scratch_bytes);
 cudaError_t launch_find_hits(const HfTable &t, int64_t nunits, void *scratch, int32_t *totals, cudaStream_t s);
 
 // Network: dense-1 partial sums [splits][n_pad][128] from patches.
