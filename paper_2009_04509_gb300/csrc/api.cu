@@ -77,6 +77,7 @@ void free_ctx(emtk_ctx *c) {
         cudaStreamSynchronize(c->copy_stream);
         cudaStreamDestroy(c->copy_stream);
     }
+    if (c->h_totals) cudaFreeHost(c->h_totals);
     for (auto &st : c->stage) {
         if (st.compute_done) cudaEventSynchronize(st.compute_done);
         if (st.buf) cudaFree(st.buf);
@@ -648,6 +649,11 @@ emtk_status emtk_find_hits(emtk_ctx *c, emtk_hitfind_request *reqs, int32_t nreq
     DeviceGuard g(c->device);
     if (!g.ok) return EMTK_ERR_CUDA;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (!c->h_totals &&
+        cudaHostAlloc((void **)&c->h_totals, sizeof(int32_t) * kMaxHfPlanes, cudaHostAllocDefault) != cudaSuccess) {
+        c->h_totals = nullptr;
+        return EMTK_ERR_OOM;
+    }
     int32_t *totals = reinterpret_cast<int32_t *>(c->ws.partials);
     void *scratch = reinterpret_cast<char *>(c->ws.partials) + 256;
     int32_t i = 0;
@@ -678,11 +684,10 @@ emtk_status emtk_find_hits(emtk_ctx *c, emtk_hitfind_request *reqs, int32_t nreq
             Prof prof(c, EMTK_KERNEL_HITFIND, s);
             e = launch_find_hits(t, U, scratch, totals, s);
         }
-        int32_t h_tot[kMaxHfPlanes];
-        if (e == cudaSuccess) e = cudaMemcpyAsync(h_tot, totals, sizeof(int32_t) * t.n, cudaMemcpyDeviceToHost, s);
+        if (e == cudaSuccess) e = cudaMemcpyAsync(c->h_totals, totals, sizeof(int32_t) * t.n, cudaMemcpyDeviceToHost, s);
         if (e == cudaSuccess) e = cudaStreamSynchronize(s);
         if (e != cudaSuccess) return cuda_status(e);
-        for (int r = 0; r < t.n; ++r) reqs[first + r].n_found = h_tot[r];
+        for (int r = 0; r < t.n; ++r) reqs[first + r].n_found = c->h_totals[r];
     }
     return EMTK_OK;
 }

@@ -162,6 +162,7 @@ struct emtk_ctx {
     } stage[2];
     cudaStream_t copy_stream = nullptr;
     uint64_t host_calls = 0;
+    int32_t *h_totals = nullptr;  // pinned: emtk_find_hits' per-plane counts (kMaxHfPlanes)
 };
 
 namespace emtk {

@@ -3,8 +3,8 @@ seeded planes.
 
 Bars: the number of hits and every integer field (wire, peak tick, start,
 end) bit-exact, the peak value bit-exact (it is an input value); the charge,
-an fp32 sum in tick order against the oracle's double sum, within
-1e-5 x sum|values| + 1e-3.  Hits found on a plane then go through
+an fp32 sum in the kernel's fixed order against the oracle's double sum,
+within 1e-5 x sum|values| + 1e-3.  Hits found on a plane then go through
 emtk_infer unchanged, and the scores match the oracle's on the oracle's
 hits.
 """
@@ -182,3 +182,67 @@ def test_found_hits_feed_inference(emtk, ctx):
     wh = np.stack([want["wire"][sel], want["tick"][sel]], 1).astype(np.int32)
     _, emu = oracle.forward(oracle.extract_patches(p.adc, p.nticks, wh), synth.he_normal_weights(0), emulate="bf16")
     assert np.abs(scores.cpu().numpy()[sel, :4] - emu).max() <= 2e-2
+
+
+def test_run_lengths_and_phases(emtk, ctx):
+    """Runs of every length 1..70 starting at every phase of the 4-tick lane
+    groups (short runs measured in registers, longer ones walked by the
+    warp), some across the 512-tick stretch edges, with tied maxima."""
+    rng = np.random.default_rng(7)
+    nt = 6000
+    adc = np.zeros((40, nt), np.float32)
+    for w in range(40):
+        t = int(rng.integers(0, 8))
+        while t < nt - 80:
+            ln = int(rng.integers(1, 71))
+            vals = rng.integers(2, 9, ln).astype(np.float32)  # small integers: many ties
+            adc[w, t:t + ln] = vals
+            t += ln + int(rng.integers(1, 40))
+    for w in range(40):  # runs across the stretch edges 512k
+        e = 512 * (1 + w % 10)
+        adc[w, e - 1 - w % 7:e + 3 + w % 5] = 5.0
+    got = gpu_find(emtk, ctx, [(adc, nt, 1.0)])[0]
+    assert check_plane(got, adc, nt, 1.0) > 2000
+
+
+def test_slots_and_overflow_mix(emtk, ctx):
+    """Units with 33..128 runs (kept in the slots) next to units with more
+    (scanned again) and units with none, in one chunk."""
+    nt = 4096
+    adc = np.zeros((64, nt), np.float32)
+    t = np.arange(nt)
+    adc[0::3] = np.where(t % 20 == 0, 3.0, 0.0)   # 103 runs per segment
+    adc[1::3] = np.where(t % 5 == 0, 3.0, 0.0)    # 410 runs per segment
+    got = gpu_find(emtk, ctx, [(adc, nt, 1.0)])[0]
+    assert check_plane(got, adc, nt, 1.0) == 22 * 205 + 21 * 820
+
+
+def test_negative_threshold_signed_zero(emtk, ctx):
+    """A negative threshold: zeros of both signs are above it and tie at the
+    peak; the first of them is the hit."""
+    adc = np.full((3, 256), -5.0, np.float32)
+    adc[0, 10:14] = [-0.0, 0.0, -1.0, 0.0]
+    adc[1, 100:140] = -0.5
+    adc[1, 120] = 0.0
+    adc[1, 125] = -0.0
+    adc[2, 0:256] = -1.0
+    got = gpu_find(emtk, ctx, [(adc, 256, -2.0)])[0]
+    check_plane(got, adc, 256, -2.0)
+    assert list(got["tick"]) == [10, 120, 0]
+    assert np.signbit(got["peak"][0])
+
+
+def test_planes_of_odd_unit_counts(emtk, ctx):
+    """Several planes in one call whose unit counts are not multiples of the
+    place kernel's 128-unit chunk, with empty planes between them."""
+    rng = np.random.default_rng(11)
+    planes = []
+    for nw, ntk in [(1, 2049), (0, 100), (130, 700), (300, 4100), (5, 0), (77, 2048), (129, 6000)]:
+        ld = max(4, (ntk + 3) // 4 * 4)
+        adc = (rng.standard_normal((nw, ld)) * 3).astype(np.float32)
+        adc[:, ntk:] = 99.0
+        planes.append((adc, ntk, 6.0))
+    got = gpu_find(emtk, ctx, planes)
+    for g, (adc, ntk, thr) in zip(got, planes):
+        check_plane(g, adc, ntk, thr)
+    assert got[1]["n"] == 0 and got[4]["n"] == 0 and got[3]["n"] > 1000
