@@ -398,6 +398,8 @@ emtk_status emtk_create(const emtk_weights *w, const emtk_options *opt, int devi
     DeviceWeights &d = c->w;
     if (e == cudaSuccess) e = upload(&d.conv_w, w->conv_w, (size_t)kK * kK * kF);
     if (e == cudaSuccess) e = upload(&d.conv_b, w->conv_b, kF);
+    std::copy(w->conv_w, w->conv_w + kK * kK * kF, d.conv_w_host);
+    std::copy(w->conv_b, w->conv_b + kF, d.conv_b_host);
     if (e == cudaSuccess) e = upload(&d.fc1_b, w->fc1_b, kN1);
     if (e == cudaSuccess) e = upload(&d.fc2_w, w->fc2_w, (size_t)kN1 * kN2);
     if (e == cudaSuccess) e = upload(&d.fc2_b, w->fc2_b, kN2);

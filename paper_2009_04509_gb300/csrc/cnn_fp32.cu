@@ -4,14 +4,18 @@
 //
 // Block = 128 hits x one segment of conv positions, 256 threads.  Per
 // position the block
-//   - computes the 128 x 48 conv activations (thread: one hit, 24 filters)
-//     from a 5-row band of the hits' patches held in shared memory (rows
-//     kept by row % 5, one new row per output row), transposed into act[48][128];
+//   - computes the 128 x 48 conv activations (thread: one hit, 24 filters;
+//     each warp one half of the filters) from a 5-row band of the hits'
+//     patches held in shared memory (rows kept by row % 5, one new row per
+//     output row), transposed into act[48][128].  The conv weights are a
+//     launch parameter, so the FMAs read them from the constant bank: one
+//     shared-memory load per tap and thread;
 //   - multiplies them into the dense-1 sums with the position's 48 x 128
 //     weights, which cp.async brought into one of two shared buffers while
 //     the previous position was computed: thread (hit group g, output group
-//     o) accumulates hits 8g..8g+7 x outputs 8o..8o+7 in 64 registers, 16
-//     FMAs per shared-memory load.
+//     o) accumulates hits 8g..8g+7 x outputs 4o..4o+3 and 64+4o..64+4o+3 in
+//     64 registers (the split keeps the weight loads free of bank
+//     conflicts), 16 FMAs per shared-memory load.
 // Segment partial sums go to partials[segment][hit][128]; the head kernel
 // adds them in segment order, so results are deterministic.
 #include "emtk_internal.h"
@@ -23,10 +27,12 @@ constexpr int kHT = 128;      // hits per block
 constexpr int kThreads = 256;
 constexpr int kBandStride = kPatch + 1;  // 49: conflict-free per-hit reads
 constexpr int kW1Pos = kF * kN1;         // 6144 weights of one position (24 KB)
-// shared memory: band[5][128][49], w1[2][48][128], act[48][128], cw[25][48], cb[48]
-constexpr int kSmemFloats = kK * kHT * kBandStride + 2 * kW1Pos + kF * kHT + kK * kK * kF + kF;
+// shared memory: band[5][128][49], w1[2][48][128], act[48][128]
+constexpr int kSmemFloats = kK * kHT * kBandStride + 2 * kW1Pos + kF * kHT;
 constexpr int kSmemBytes = kSmemFloats * 4;
 static_assert(kSmemBytes <= 232448, "shared memory budget");
+static_assert(kW1Pos % (4 * kThreads) == 0 && kHT % 32 == 0 && kThreads == 2 * kHT && kThreads / 16 * 8 == kHT,
+              "thread layout: two conv filter halves of kHT hits; 16 threads per 8 hits in dense-1");
 
 __device__ __forceinline__ void cp_async16(float *smem_dst, const float *gmem_src) {
     const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(smem_dst));
@@ -62,28 +68,49 @@ __device__ __forceinline__ void load_band_row(float *band, const float *__restri
     }
 }
 
+// The conv weights [25][48] and bias [48], passed by value.
+struct ConvParams {
+    float w[kK * kK * kF];
+    float b[kF];
+};
+
+// Conv + ReLU of hit `hit` at position (y, x), filters F0 .. F0+23, into act.
+template <int F0>
+__device__ __forceinline__ void conv_half(const ConvParams &cp, const float *band, int y, int x, int hit, float *act) {
+    float s[24];
+#pragma unroll
+    for (int f = 0; f < 24; ++f) s[f] = cp.b[F0 + f];
+#pragma unroll
+    for (int i = 0; i < kK; ++i) {
+        const float *row = band + ((y + i) % kK) * kHT * kBandStride + hit * kBandStride + x;
+#pragma unroll
+        for (int j = 0; j < kK; ++j) {
+            const float v = row[j];
+#pragma unroll
+            for (int f = 0; f < 24; ++f) s[f] = fmaf(v, cp.w[(i * kK + j) * kF + F0 + f], s[f]);
+        }
+    }
+#pragma unroll
+    for (int f = 0; f < 24; ++f) act[(F0 + f) * kHT + hit] = fmaxf(s[f], 0.0f);
+}
+
 __global__ void __launch_bounds__(kThreads, 1) cnn_fp32_kernel(const float *__restrict__ patches, int n,
-                                                               const float *__restrict__ conv_w,
-                                                               const float *__restrict__ conv_b,
+                                                               const __grid_constant__ ConvParams cp,
                                                                const float *__restrict__ fc1_w, int splits,
                                                                float *__restrict__ partials, int n_pad) {
     extern __shared__ float4 smem_f4[];
     float *band = reinterpret_cast<float *>(smem_f4);  // [5][128][49]
     float *w1 = band + kK * kHT * kBandStride;          // [2][48][128]
     float *act = w1 + 2 * kW1Pos;                       // [48][128]
-    float *cw = act + kF * kHT;                         // [25][48]
-    float *cb = cw + kK * kK * kF;                      // [48]
 
     const int tid = threadIdx.x;
     const int hit0 = blockIdx.x * kHT;
     const int seg = blockIdx.y;
     const int p_begin = (int)((int64_t)seg * kPos / splits);
     const int p_end = (int)((int64_t)(seg + 1) * kPos / splits);
-    for (int i = tid; i < kK * kK * kF; i += kThreads) cw[i] = conv_w[i];
-    for (int i = tid; i < kF; i += kThreads) cb[i] = conv_b[i];
 
-    const int g = tid >> 4, o = tid & 15;        // dense-1: hits 8g.., outputs 8o..
-    const int ch = tid >> 1, f0 = (tid & 1) * 24;  // conv: hit ch, filters f0..f0+23
+    const int g = tid >> 4, o = tid & 15;  // dense-1: hits 8g.., outputs 4o.. and 64+4o..
+    const int ch = tid & (kHT - 1);        // conv: hit ch, filter half tid / 128 (one per warp)
     float acc[8][8];
 #pragma unroll
     for (int i = 0; i < 8; ++i)
@@ -103,23 +130,11 @@ __global__ void __launch_bounds__(kThreads, 1) cnn_fp32_kernel(const float *__re
             band_y = y;
             __syncthreads();
         }
-        // conv + ReLU of hit ch, filters f0 .. f0+23, transposed into act
-        float s[24];
-#pragma unroll
-        for (int f = 0; f < 24; ++f) s[f] = cb[f0 + f];
-#pragma unroll
-        for (int i = 0; i < kK; ++i) {
-            const float *row = band + ((y + i) % kK) * kHT * kBandStride + ch * kBandStride + x;
-#pragma unroll
-            for (int j = 0; j < kK; ++j) {
-                const float v = row[j];
-                const float *wrow = cw + (i * kK + j) * kF + f0;
-#pragma unroll
-                for (int f = 0; f < 24; ++f) s[f] = fmaf(v, wrow[f], s[f]);
-            }
-        }
-#pragma unroll
-        for (int f = 0; f < 24; ++f) act[(f0 + f) * kHT + ch] = fmaxf(s[f], 0.0f);
+        // conv + ReLU, transposed into act
+        if (tid < kHT)
+            conv_half<0>(cp, band, y, x, ch, act);
+        else
+            conv_half<24>(cp, band, y, x, ch, act);
         cp_async_wait_prev();  // this position's weights have landed
         __syncthreads();
         // dense-1: 8 hits x 8 outputs per thread
@@ -128,8 +143,8 @@ __global__ void __launch_bounds__(kThreads, 1) cnn_fp32_kernel(const float *__re
         for (int c = 0; c < kF; ++c) {
             const float4 a0 = *reinterpret_cast<const float4 *>(act + c * kHT + 8 * g);
             const float4 a1 = *reinterpret_cast<const float4 *>(act + c * kHT + 8 * g + 4);
-            const float4 b0 = *reinterpret_cast<const float4 *>(wp + c * kN1 + 8 * o);
-            const float4 b1 = *reinterpret_cast<const float4 *>(wp + c * kN1 + 8 * o + 4);
+            const float4 b0 = *reinterpret_cast<const float4 *>(wp + c * kN1 + 4 * o);
+            const float4 b1 = *reinterpret_cast<const float4 *>(wp + c * kN1 + 64 + 4 * o);
             const float a[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
             const float b[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
 #pragma unroll
@@ -143,9 +158,9 @@ __global__ void __launch_bounds__(kThreads, 1) cnn_fp32_kernel(const float *__re
     for (int i = 0; i < 8; ++i) {
         const int gh = hit0 + 8 * g + i;
         if (gh < n) {
-            float *dst = partials + ((int64_t)seg * n_pad + gh) * kN1 + 8 * o;
-            reinterpret_cast<float4 *>(dst)[0] = make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
-            reinterpret_cast<float4 *>(dst)[1] = make_float4(acc[i][4], acc[i][5], acc[i][6], acc[i][7]);
+            float *dst = partials + ((int64_t)seg * n_pad + gh) * kN1;
+            reinterpret_cast<float4 *>(dst + 4 * o)[0] = make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
+            reinterpret_cast<float4 *>(dst + 64 + 4 * o)[0] = make_float4(acc[i][4], acc[i][5], acc[i][6], acc[i][7]);
         }
     }
 }
@@ -168,8 +183,11 @@ int choose_splits_fp32(int n, int sm_count, int max_splits) {
 cudaError_t launch_cnn_fp32(const DeviceWeights &w, const float *patches, int32_t n, int splits, float *partials,
                             int n_pad, cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
+    ConvParams cp;
+    for (int i = 0; i < kK * kK * kF; ++i) cp.w[i] = w.conv_w_host[i];
+    for (int i = 0; i < kF; ++i) cp.b[i] = w.conv_b_host[i];
     dim3 grid((n + kHT - 1) / kHT, splits);
-    cnn_fp32_kernel<<<grid, kThreads, kSmemBytes, s>>>(patches, n, w.conv_w, w.conv_b, w.fc1_w, splits, partials, n_pad);
+    cnn_fp32_kernel<<<grid, kThreads, kSmemBytes, s>>>(patches, n, cp, w.fc1_w, splits, partials, n_pad);
     return cudaGetLastError();
 }
 

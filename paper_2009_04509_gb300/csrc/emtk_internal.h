@@ -128,6 +128,10 @@ struct DeviceWeights {
     void *w1_tmap = nullptr;       // host copy of the TMA descriptor (CUtensorMap, 128 B)
     float fc1_scale = 1.0f;        // dense-1 sums are scaled by this before the bias (EMTK_FP8: 1/(s_a s_w))
     float fc1_w_scale = 1.0f;      // EMTK_FP8: s_w, the power of two the weights were scaled by
+    // host copy of the conv weights [25][48] and bias [48]: the fp32 kernel takes
+    // them as a launch parameter (constant bank)
+    float conv_w_host[kK * kK * kF] = {};
+    float conv_b_host[kF] = {};
 };
 
 // Operand formats of the tensor-core kernel.
