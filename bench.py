@@ -376,7 +376,14 @@ def main():
                        "bytes_read": union, "bytes_written": patch_bytes,
                        "kernels": "interval_image_kernel + " + ("gather_kernel" if args.precision == "fp32"
                                                                else "hit_desc_kernel"),
-                       "ms_per_step": cut_ms},
+                       "ms_per_step": cut_ms,
+                       # the cut's output counted as patches (16-bit: 4,608 B per hit), as the
+                       # hot-path scope defines K1; the tensor path never writes them, so the
+                       # frac above (union read + interval image written) is the stricter one
+                       "with_logical_patch_write": {
+                           "algorithmic_bytes": union + nhits * 48 * 48 * (4 if args.precision == "fp32" else 2),
+                           "frac": (union + nhits * 48 * 48 * (4 if args.precision == "fp32" else 2))
+                           / (cut_ms / 1e3) / 1e9 / peaks["hbm"]}},
         "step_ms_stats": {"median": statistics.median(step_ms), "min": min(step_ms), "max": max(step_ms),
                           "mean": total_ms / args.steps, "n": len(step_ms)},
         "kernel_ms_per_step": {k: v / args.steps for k, v in kms.items()},

@@ -206,6 +206,18 @@ def test_tile_edges(emtk, ctx_factory, weights, n):
     check_invariants(got)
 
 
+@pytest.mark.parametrize("n", [1, 127, 129, 383, 2049])
+def test_fp32_tile_edges(emtk, ctx_factory, weights, n):
+    """The fp32 path at hit counts off its 128-hit tile; the number of K
+    splits it picks changes with the count (one split per ~16 positions up
+    to about four waves of blocks)."""
+    plane = synth.single_plane(seed=8, nhits=n, nticks=1200)
+    got = run_infer(emtk, ctx_factory(weights, "fp32"), plane)
+    _, ref = oracle.forward(oracle.extract_patches(plane.adc, plane.nticks, plane.hits), weights)
+    assert np.abs(got[:, :4] - ref).max() <= TOL_FP32
+    check_invariants(got)
+
+
 def test_edge_hits_network(emtk, ctx_factory, weights):
     """Hits on plane corners, outside it and duplicated run through the network."""
     rng = np.random.default_rng(6)
@@ -318,3 +330,26 @@ def test_full_event_sampled(emtk, ctx_factory, weights):
     emtk.emtk_extract_patches(ctx, dev(p.adc), p.nticks, dev(p.hits[idx]), out, "f32")
     want = oracle.extract_patches(p.adc, p.nticks, p.hits[idx])
     assert np.array_equal(out.cpu().numpy().view(np.uint32), want.view(np.uint32))
+
+
+def test_fp32_full_event_sampled(emtk, ctx_factory, weights):
+    """The fp32 path on the full 18-plane event (60,000 hits) in one batched
+    call, as `bench.py --precision fp32` runs it; sampled hits against the
+    fp64 oracle at the fp32 bar, every hit against the invariants."""
+    planes = synth.full_event(seed=0)
+    ctx = ctx_factory(weights, "fp32")
+    items, outs = [], []
+    for p in planes:
+        s = torch.full((p.nhits, 8), float("nan"), device="cuda")
+        items.append((dev(p.adc), p.nticks, dev(p.hits), s))
+        outs.append(s)
+    emtk.emtk_infer_batch(ctx, items)
+    assert emtk.emtk_check(ctx) == emtk.EMTK_OK
+    got = [s.cpu().numpy().astype(np.float64) for s in outs]
+    check_invariants(np.concatenate(got))
+    rng = np.random.default_rng(12)
+    per = 96 // len(planes) + 1
+    for p, g in zip(planes, got):
+        idx = rng.choice(p.nhits, per, replace=False)
+        _, ref = oracle.forward(oracle.extract_patches(p.adc, p.nticks, p.hits[idx]), weights)
+        assert np.abs(g[idx, :4] - ref).max() <= TOL_FP32
