@@ -416,6 +416,7 @@ emtk_status emtk_create(const emtk_weights *w, const emtk_options *opt, int devi
             if (e == cudaSuccess) e = init_fp32_kernel_attrs();
         }
     }
+    if (e == cudaSuccess) e = init_head_kernel_attrs();
     if (e == cudaSuccess) e = alloc_workspace(c, true);
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
     if (e != cudaSuccess) {

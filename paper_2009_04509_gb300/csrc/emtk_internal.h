@@ -221,6 +221,7 @@ cudaError_t launch_head(const DeviceWeights &w, const float *partials, int split
 
 // Kernel attributes (dynamic shared memory), set once per device at create.
 cudaError_t init_fp32_kernel_attrs();
+cudaError_t init_head_kernel_attrs();
 cudaError_t init_tc_kernel_attrs();
 
 // Host helpers for the tensor-core weights (cnn_tc.cu).

@@ -12,6 +12,20 @@ namespace emtk {
 namespace {
 
 constexpr int kThreadsHead = 128;
+
+// The dense-2 weights [128][32] into shared memory (16-byte aligned): every
+// load issued before the first store, so that staging costs one round trip.
+template <int kThreads>
+__device__ __forceinline__ void stage_w2(float *w2, const float *__restrict__ fc2_w) {
+    constexpr int kN4 = kN1 * kN2 / 4;
+    static_assert(kN4 % kThreads == 0, "whole float4s per thread");
+    float4 v[kN4 / kThreads];
+#pragma unroll
+    for (int k = 0; k < kN4 / kThreads; ++k)
+        v[k] = __ldg(reinterpret_cast<const float4 *>(fc2_w) + threadIdx.x + k * kThreads);
+#pragma unroll
+    for (int k = 0; k < kN4 / kThreads; ++k) reinterpret_cast<float4 *>(w2)[threadIdx.x + k * kThreads] = v[k];
+}
 constexpr int kManyRows = 4;  // above this many partial rows per hit, reduce them with a warp per hit
 
 __global__ void __launch_bounds__(kThreadsHead) head_kernel(const float *__restrict__ partials, int splits, int G,
@@ -28,7 +42,7 @@ __global__ void __launch_bounds__(kThreadsHead) head_kernel(const float *__restr
     __shared__ __align__(16) float wc[kN2][kNC + 1];
     __shared__ __align__(16) float b1[kN1];
     __shared__ float b2[kN2];
-    for (int i = threadIdx.x; i < kN1 * kN2; i += blockDim.x) w2[i / kN2][i % kN2] = fc2_w[i];
+    stage_w2<kThreadsHead>(&w2[0][0], fc2_w);
     for (int i = threadIdx.x; i < kN2 * kNC; i += blockDim.x) wc[i / kNC][i % kNC] = cls_w[i];
     for (int i = threadIdx.x; i < kN2; i += blockDim.x) {
         wc[i][kNC] = mic_w[i];
@@ -130,7 +144,7 @@ __global__ void __launch_bounds__(kThreadsRows) head_rows_kernel(const float *__
     __shared__ __align__(16) float w2[kN1][kN2];
     __shared__ __align__(16) float wc[kN2][kNC + 1];
     __shared__ float b2[kN2];
-    for (int i = threadIdx.x; i < kN1 * kN2; i += blockDim.x) w2[i / kN2][i % kN2] = fc2_w[i];
+    stage_w2<kThreadsRows>(&w2[0][0], fc2_w);
     for (int i = threadIdx.x; i < kN2 * kNC; i += blockDim.x) wc[i / kNC][i % kNC] = cls_w[i];
     for (int i = threadIdx.x; i < kN2; i += blockDim.x) {
         wc[i][kNC] = mic_w[i];
@@ -151,8 +165,23 @@ __global__ void __launch_bounds__(kThreadsRows) head_rows_kernel(const float *__
         }
         const float4 *p = reinterpret_cast<const float4 *>(partials + h * kN1) + lane;
         float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 4
-        for (int r = 0; r < rows; ++r) {  // rows in order: the same sum as head_kernel
+        // rows in order (the same sum as head_kernel), loaded 16 at a time so that a
+        // hit with many rows waits for a few round trips, not one per row
+        constexpr int kDepth = 16;
+        int r = 0;
+        for (; r + kDepth <= rows; r += kDepth) {
+            float4 v[kDepth];
+#pragma unroll
+            for (int k = 0; k < kDepth; ++k) v[k] = p[(r + k) * row_stride];
+#pragma unroll
+            for (int k = 0; k < kDepth; ++k) {
+                a.x += v[k].x;
+                a.y += v[k].y;
+                a.z += v[k].z;
+                a.w += v[k].w;
+            }
+        }
+        for (; r < rows; ++r) {
             const float4 v = p[r * row_stride];
             a.x += v.x;
             a.y += v.y;
@@ -211,7 +240,143 @@ __global__ void __launch_bounds__(kThreadsRows) head_rows_kernel(const float *__
     }
 }
 
+// The tail of a large launch with few partial rows per hit: one CTA per
+// 128-hit tile (every hit of a tile has the same rows), 256 threads.
+//   1. warp w sums the rows of hits 16w .. 16w+15, lane l taking dense-1
+//      outputs l, l+32, l+64, l+96 (four coalesced 128-byte reads per row),
+//      and writes bias + ReLU transposed, h1t[k][hit];
+//   2. dense-2: thread (hit group tid % 32, output group tid / 32) keeps 4
+//      hits x 4 outputs, reading 4 activations and 4 weights (a broadcast)
+//      per input k; sums to h2s[hit][j];
+//   3. a thread per hit: ReLU, the heads.
+// Sums run in the same order as head_kernel's (rows in order; k in order for
+// every output), so all three kernels give the same bits.
+constexpr int kTileHits = 128;
+constexpr int kThreadsTile = 256;
+constexpr int kH1tStride = kTileHits + 4;  // rows of h1t: 16-byte aligned, banks shifted per k
+
+__global__ void __launch_bounds__(kThreadsTile) head_tile_kernel(const float *__restrict__ partials, int splits,
+                                                                int G, int n_pad, int32_t n, float s1,
+                                                                const float *__restrict__ fc1_b,
+                                                                const float *__restrict__ fc2_w,
+                                                                const float *__restrict__ fc2_b,
+                                                                const float *__restrict__ cls_w,
+                                                                const float *__restrict__ cls_b,
+                                                                const float *__restrict__ mic_w,
+                                                                const float *__restrict__ mic_b, float *const *dest,
+                                                                int debug_logits) {
+    extern __shared__ __align__(16) float tsm[];
+    float *h1t = tsm;                                    // [kN1][kH1tStride]
+    float *w2 = h1t + kN1 * kH1tStride;                  // [kN1][kN2]
+    float *h2s = w2 + kN1 * kN2;                         // [kTileHits][kN2 + 1]
+    __shared__ __align__(16) float wc[kN2][kNC + 1];
+    __shared__ float b2[kN2];
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    stage_w2<kThreadsTile>(w2, fc2_w);
+    for (int i = tid; i < kN2 * kNC; i += kThreadsTile) wc[i / kNC][i % kNC] = cls_w[i];
+    for (int i = tid; i < kN2; i += kThreadsTile) {
+        wc[i][kNC] = mic_w[i];
+        b2[i] = fc2_b[i];
+    }
+    const int64_t h0 = (int64_t)blockIdx.x * kTileHits;
+    int rows = splits;
+    if (G > 0) {
+        const int64_t units = (int64_t)((n + 127) / 128) * kQuads;
+        const int64_t tile = h0 >> 7;
+        rows = cta_of_unit(tile * kQuads + kQuads - 1, units, G) - cta_of_unit(tile * kQuads, units, G) + 1;
+    }
+    const int64_t row_stride = (int64_t)n_pad * kN1;  // floats between partial rows
+    float bb[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) bb[e] = fc1_b[lane + 32 * e];
+    // the warp's hits warp, warp + 8, ...: eight at a time, so that 32 loads per lane
+    // are in flight before the first is used
+    constexpr int kBatch = 8;
+    for (int j0 = warp; j0 < kTileHits; j0 += kBatch * (kThreadsTile / 32)) {
+        float a[kBatch][4];
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {
+            const int64_t h = h0 + j0 + u * (kThreadsTile / 32);
+            const float *p = partials + (h < n ? h : 0) * kN1 + lane;
+#pragma unroll
+            for (int e = 0; e < 4; ++e) a[u][e] = h < n ? p[32 * e] : 0.f;
+        }
+        for (int r = 1; r < rows; ++r) {
+#pragma unroll
+            for (int u = 0; u < kBatch; ++u) {
+                const int64_t h = h0 + j0 + u * (kThreadsTile / 32);
+                const float *p = partials + (h < n ? h : 0) * kN1 + lane + r * row_stride;
+#pragma unroll
+                for (int e = 0; e < 4; ++e) a[u][e] += h < n ? p[32 * e] : 0.f;
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u)
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+                h1t[(lane + 32 * e) * kH1tStride + j0 + u * (kThreadsTile / 32)] = fmaxf(fmaf(a[u][e], s1, bb[e]), 0.f);
+    }
+    __syncthreads();
+    {
+        const int hg = lane, og = warp;  // hits 4hg .. 4hg+3, outputs 4og .. 4og+3
+        float acc[4][4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int q = 0; q < 4; ++q) acc[i][q] = b2[4 * og + q];
+#pragma unroll 4
+        for (int k = 0; k < kN1; ++k) {
+            const float4 x = *reinterpret_cast<const float4 *>(h1t + k * kH1tStride + 4 * hg);
+            const float4 wv = *reinterpret_cast<const float4 *>(w2 + k * kN2 + 4 * og);
+            const float xs[4] = {x.x, x.y, x.z, x.w};
+            const float ws[4] = {wv.x, wv.y, wv.z, wv.w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int q = 0; q < 4; ++q) acc[i][q] = fmaf(xs[i], ws[q], acc[i][q]);
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int q = 0; q < 4; ++q) h2s[(4 * hg + i) * (kN2 + 1) + 4 * og + q] = acc[i][q];
+    }
+    __syncthreads();
+    if (tid >= kTileHits) return;
+    const int64_t h = h0 + tid;
+    if (h >= n) return;
+    const float *h2 = h2s + tid * (kN2 + 1);
+    float z[kNC + 1] = {cls_b[0], cls_b[1], cls_b[2], mic_b[0]};
+#pragma unroll
+    for (int j = 0; j < kN2; ++j) {
+        const float v = fmaxf(h2[j], 0.f);
+        const float4 wv = *reinterpret_cast<const float4 *>(&wc[j][0]);
+        z[0] = fmaf(v, wv.x, z[0]);
+        z[1] = fmaf(v, wv.y, z[1]);
+        z[2] = fmaf(v, wv.z, z[2]);
+        z[3] = fmaf(v, wv.w, z[3]);
+    }
+    const float m = fmaxf(fmaxf(z[0], z[1]), z[2]);
+    const float e0 = expf(z[0] - m), e1 = expf(z[1] - m), e2 = expf(z[2] - m);
+    const float sum = e0 + e1 + e2;
+    float *out = dest[h];
+    out[0] = e0 / sum;
+    out[1] = e1 / sum;
+    out[2] = e2 / sum;
+    out[3] = 1.0f / (1.0f + expf(-z[kNC]));
+    if (debug_logits) {
+        out[4] = z[0];
+        out[5] = z[1];
+        out[6] = z[2];
+        out[7] = z[3];
+    }
+}
+constexpr int kTileSmem = (kN1 * kH1tStride + kN1 * kN2 + kTileHits * (kN2 + 1)) * 4;
+
 }  // namespace
+
+cudaError_t init_head_kernel_attrs() {
+    return cudaFuncSetAttribute(head_tile_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kTileSmem);
+}
 
 cudaError_t launch_head(const DeviceWeights &w, const float *partials, int splits, int G, int n_pad, int32_t n,
                         float *const *dest, int debug_logits, cudaStream_t s) {
@@ -227,6 +392,12 @@ cudaError_t launch_head(const DeviceWeights &w, const float *partials, int split
             head_rows_kernel<32><<<(n + 31) / 32, kThreadsRows, 0, s>>>(
                 partials, splits, G, n_pad, n, w.fc1_scale, w.fc1_b, w.fc2_w, w.fc2_b, w.cls_w, w.cls_b, w.mic_w,
                 w.mic_b, dest, debug_logits);
+        return cudaGetLastError();
+    }
+    if (n > kSmallLaunch) {
+        head_tile_kernel<<<(n + kTileHits - 1) / kTileHits, kThreadsTile, kTileSmem, s>>>(
+            partials, splits, G, n_pad, n, w.fc1_scale, w.fc1_b, w.fc2_w, w.fc2_b, w.cls_w, w.cls_b, w.mic_w,
+            w.mic_b, dest, debug_logits);
         return cudaGetLastError();
     }
     head_kernel<<<(n + kThreadsHead - 1) / kThreadsHead, kThreadsHead, 0, s>>>(
