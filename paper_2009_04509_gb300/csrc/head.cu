@@ -1,11 +1,17 @@
 // Network tail (Sec. 2.2), fp32: sum of the dense-1 partial-sum rows in row
 // order, times the dense-1 scale s1 (1, or the inverse of the operand scales
-// of the e4m3 path), + bias + ReLU, dense 128->32 + ReLU, the 3-way softmax head (track,
-// em, none) and the Michel sigmoid head.  One thread per hit: the thread
-// streams its dense-1 outputs four at a time and folds each into the 32
-// dense-2 sums at once (weights broadcast from shared memory), so only the
-// 32 sums stay live.  The rows of a hit are the K-splits of the fp32 path,
-// or the stream-K CTAs that shared its tile.
+// of the e4m3 path), + bias + ReLU, dense 128->32 + ReLU, the 3-way softmax
+// head (track, em, none) and the Michel sigmoid head.  The rows of a hit are
+// the K-splits of the fp32 path, or the stream-K CTAs that shared its tile.
+// Three kernels, chosen by launch_head, with the same sums in the same order
+// (so the same bits):
+//   head_kernel       small launches with few rows: a thread per hit streams
+//                     its dense-1 outputs four at a time into the 32 dense-2
+//                     sums (weights broadcast from shared memory);
+//   head_rows_kernel  many rows per hit (small launches spread each tile
+//                     over many CTAs): a warp per hit sums the rows, 16 deep;
+//   head_tile_kernel  large launches: one CTA per 128-hit tile (coalesced
+//                     row sums, a register-tiled dense-2).
 #include "emtk_internal.h"
 
 namespace emtk {

@@ -16,7 +16,8 @@
 //                    that lane from registers; a run that goes past them is
 //                    walked by the whole warp, 32 ticks per step, past the
 //                    segment's end if it goes on (the stretch's samples from
-//                    a shared-memory copy, later ticks from global memory).  The warp keeps the unit's first kRunSlots runs in
+//                    a shared-memory copy, later ticks from global memory).
+//                    The warp keeps the unit's first kRunSlots runs in
 //                    scratch slots, writes its run count and adds it to its
 //                    chunk's sum (chunks: kHfChunk consecutive units of one
 //                    plane);
@@ -29,11 +30,12 @@
 //                    threads write consecutive hits.  A unit with more runs
 //                    than slots is scanned again by a warp and written
 //                    directly.  The plane's last unit writes its total.
-// The plane is read once from HBM (plus units with more than kRunSlots runs).
-// No kernel waits on another CTA.  Outputs are ordered by wire, then tick,
-// whatever the launch shape.  The samples are read with the streaming
-// (evict-first) hint: each is used once, apart from walks of runs that go
-// past a lane's 4 ticks.
+// A memset of the chunk sums precedes the two kernels.  The plane is read
+// once from HBM (plus units with more than kRunSlots runs).  No kernel waits
+// on another CTA.  Outputs are ordered by wire, then tick, whatever the
+// launch shape.  The samples are read with the streaming (evict-first) hint:
+// each is used once, apart from walks of runs that go past a lane's 4 ticks,
+// which read the stretch's shared-memory copy.
 #include <cmath>
 
 #include "emtk_internal.h"
