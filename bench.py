@@ -374,8 +374,8 @@ def main():
         "extraction": {"bound": "hbm", "achieved": cut_gbs, "peak": peaks["hbm"], "unit": "GB/s",
                        "frac": cut_gbs / peaks["hbm"], "algorithmic_bytes": union + patch_bytes,
                        "bytes_read": union, "bytes_written": patch_bytes,
-                       "kernels": "interval_image_kernel + " + ("gather_kernel" if args.precision == "fp32"
-                                                               else "hit_desc_kernel"),
+                       "kernels": "interval_image_kernel + gather_kernel" if args.precision == "fp32"
+                       else "interval_desc_kernel (images + window descriptors, one launch)",
                        "ms_per_step": cut_ms,
                        # the cut's output counted as patches (16-bit: 4,608 B per hit), as the
                        # hot-path scope defines K1; the tensor path never writes them, so the

@@ -290,7 +290,9 @@ typedef struct {
  * once the results are complete: it synchronises `stream` to fill each
  * n_found.
  * EMTK_ERR_ARG for negative sizes, ld < nticks, capacity > 0 with a NULL
- * d_hits, or a plane holding more than 2^31 - 1 possible runs; EMTK_ERR_ALIGN
+ * d_hits, a plane holding more than 2^31 - 1 possible runs, or a plane of
+ * more 2048-tick wire segments than the workspace's scratch holds (about
+ * 104,000, some 214 M samples, for the default workspace); EMTK_ERR_ALIGN
  * as for emtk_infer.  The context's workspace serves as scratch, so calls on
  * one context must not overlap with each other or with its inference calls
  * on another stream. */

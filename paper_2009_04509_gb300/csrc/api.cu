@@ -243,8 +243,12 @@ emtk_status run_requests(emtk_ctx *c, const emtk_request *reqs, int32_t nreq, cu
         if (st != EMTK_OK) break;
         cudaError_t e;
         {
+            // the tensor-core kernel reads the windows straight from the images; the
+            // first chunk's window descriptors are built in the same launch
+            const DescJob job{0, (int32_t)std::min<int64_t>(c->max_hits, hits), c->ws.hdesc, c->ws.dest,
+                              out_stride(c)};
             Prof prof(c, EMTK_KERNEL_INTERVALS, s);
-            e = launch_interval_images(*t, c->ws.dimg, fmt, s);
+            e = launch_interval_images(*t, c->ws.dimg, fmt, s, tc ? &job : nullptr);
         }
         if (e != cudaSuccess) {
             st = cuda_status(e);
@@ -252,12 +256,12 @@ emtk_status run_requests(emtk_ctx *c, const emtk_request *reqs, int32_t nreq, cu
         }
         for (int64_t g0 = 0; g0 < hits && st == EMTK_OK; g0 += c->max_hits) {
             const int32_t cnt = (int32_t)std::min<int64_t>(c->max_hits, hits - g0);
-            {
+            if (tc && g0 > 0) {
                 Prof prof(c, EMTK_KERNEL_GATHER, s);
-                if (tc)  // the tensor-core kernel reads the windows straight from the images
-                    e = launch_hit_desc(*t, g0, cnt, c->ws.hdesc, c->ws.dest, out_stride(c), s);
-                else
-                    e = launch_gather(*t, c->ws.dimg, fmt, g0, cnt, c->ws.patches, c->ws.dest, out_stride(c), s);
+                e = launch_hit_desc(*t, g0, cnt, c->ws.hdesc, c->ws.dest, out_stride(c), s);
+            } else if (!tc) {
+                Prof prof(c, EMTK_KERNEL_GATHER, s);
+                e = launch_gather(*t, c->ws.dimg, fmt, g0, cnt, c->ws.patches, c->ws.dest, out_stride(c), s);
             }
             if (e != cudaSuccess) {
                 st = cuda_status(e);

@@ -182,7 +182,17 @@ void destroy_lane_ctx(emtk_ctx *c);
 // ---- kernels launched from the API (each returns cudaGetLastError()).
 // Interval images of every request plane: img[r] is [nwires][nint] of the
 // patch format (fp32 or 16-bit), at element offset r.d_off.
-cudaError_t launch_interval_images(const ReqTable &t, void *dimg, emtk_patch_format fmt, cudaStream_t s);
+// Window descriptors to build along with the images (tensor-core path): hits
+// g0 .. g0 + count - 1 of the table into desc[0 ..] and dest[0 ..].
+struct DescJob {
+    int64_t g0;
+    int32_t count;
+    HitDesc *desc;
+    float **dest;
+    int out_stride;
+};
+cudaError_t launch_interval_images(const ReqTable &t, void *dimg, emtk_patch_format fmt, cudaStream_t s,
+                                   const DescJob *job = nullptr);
 // Patches of hits [g0, g0+count) of the concatenated list (global index).
 // Writes patches[(g - g0)] and, if dest != null, dest[g - g0] = output row.
 cudaError_t launch_gather(const ReqTable &t, const void *dimg, emtk_patch_format fmt, int64_t g0,

@@ -60,12 +60,11 @@ __device__ __forceinline__ void store2(void *base, int64_t idx, float v0, float 
 // One thread = two consecutive image columns of one image row; inside the
 // plane that is two intervals of one wire (12 ticks = 48 bytes, 16-byte
 // aligned because ld % 4 == 0, the plane is 16-byte aligned and the halo is
-// even), outside it (the zero halo, the pitch padding) zeros.  grid.y =
-// request; the pitch and the image offset are even, so the pair store is
-// aligned too.
+// even), outside it (the zero halo, the pitch padding) zeros.  The image
+// of request r, grid-stride over its column pairs along x; the pitch and the
+// image offset are even, so the pair store is aligned too.
 template <int FMT>
-__global__ void __launch_bounds__(256) interval_image_kernel(const __grid_constant__ ReqTable t, void *img) {
-    const ReqDesc &r = t.r[blockIdx.y];
+__device__ __forceinline__ void interval_request(const ReqDesc &r, void *img) {
     if (r.nwires == 0) return;
     const int npairs = r.pitch >> 1;
     const int rows = r.nwires + 2 * r.halo;
@@ -90,6 +89,12 @@ __global__ void __launch_bounds__(256) interval_image_kernel(const __grid_consta
         }
         store2<FMT>(img, r.d_off + (int64_t)wr * r.pitch + cb, v0, v1, true);
     }
+}
+
+// grid.y = request.
+template <int FMT>
+__global__ void __launch_bounds__(256) interval_image_kernel(const __grid_constant__ ReqTable t, void *img) {
+    interval_request<FMT>(t.r[blockIdx.y], img);
 }
 
 template <int FMT>
@@ -173,10 +178,9 @@ __global__ void convert_kernel(const float *src, void *dst, int64_t n) {
     }
 }
 
-__global__ void hit_desc_kernel(const __grid_constant__ ReqTable t, int64_t g0, int32_t count, HitDesc *desc,
-                                float **dest, int out_stride) {
-    const int64_t local = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (local >= count) return;
+// The window descriptor of hit g0 + local of the table (and its output row).
+__device__ __forceinline__ void hit_desc_one(const ReqTable &t, int64_t g0, int64_t local, HitDesc *desc,
+                                             float **dest, int out_stride) {
     const int64_t g = g0 + local;
     const ReqDesc &r = t.r[find_request(t, g)];
     const int64_t hloc = g - r.hit_begin;
@@ -197,6 +201,28 @@ __global__ void hit_desc_kernel(const __grid_constant__ ReqTable t, int64_t g0, 
     if (dest != nullptr) dest[local] = r.scores + hloc * out_stride;
 }
 
+__global__ void hit_desc_kernel(const __grid_constant__ ReqTable t, int64_t g0, int32_t count, HitDesc *desc,
+                                float **dest, int out_stride) {
+    const int64_t local = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (local < count) hit_desc_one(t, g0, local, desc, dest, out_stride);
+}
+
+// The images (grid rows 0 .. t.n - 1) and, in one more grid row, the window
+// descriptors of hits g0 .. g0 + count - 1: the descriptors' few bytes ride
+// along with the images' stream instead of taking a launch of their own.
+template <int FMT>
+__global__ void __launch_bounds__(256) interval_desc_kernel(const __grid_constant__ ReqTable t, void *img, int64_t g0,
+                                                            int32_t count, HitDesc *desc, float **dest,
+                                                            int out_stride) {
+    if ((int)blockIdx.y < t.n) {
+        interval_request<FMT>(t.r[blockIdx.y], img);
+        return;
+    }
+    for (int64_t local = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; local < count;
+         local += (int64_t)gridDim.x * blockDim.x)
+        hit_desc_one(t, g0, local, desc, dest, out_stride);
+}
+
 __global__ void fill_dest_kernel(float *scores, int stride, float **dest, int32_t n) {
     const int i = blockIdx.x * blockDim.x + threadIdx.x;
     if (i < n) dest[i] = scores + (int64_t)i * stride;
@@ -204,11 +230,30 @@ __global__ void fill_dest_kernel(float *scores, int stride, float **dest, int32_
 
 }  // namespace
 
-cudaError_t launch_interval_images(const ReqTable &t, void *dimg, emtk_patch_format fmt, cudaStream_t s) {
+cudaError_t launch_interval_images(const ReqTable &t, void *dimg, emtk_patch_format fmt, cudaStream_t s,
+                                   const DescJob *job) {
     int64_t most = 0;
     for (int i = 0; i < t.n; ++i) {
         const int64_t w = t.r[i].nwires ? (int64_t)(t.r[i].nwires + 2 * t.r[i].halo) * (t.r[i].pitch / 2) : 0;
         most = w > most ? w : most;
+    }
+    if (job != nullptr && job->count > 0) {
+        if (most == 0 || t.n == 0)  // no image to cut: the descriptors alone
+            return launch_hit_desc(t, job->g0, job->count, job->desc, job->dest, job->out_stride, s);
+        const int64_t want = most > job->count ? most : job->count;
+        int64_t bx = (want + 255) / 256;
+        if (bx > 4096) bx = 4096;
+        dim3 grid((unsigned)bx, (unsigned)t.n + 1);
+        if (fmt == EMTK_PATCH_F32)
+            interval_desc_kernel<EMTK_PATCH_F32><<<grid, 256, 0, s>>>(t, dimg, job->g0, job->count, job->desc,
+                                                                      job->dest, job->out_stride);
+        else if (fmt == EMTK_PATCH_BF16)
+            interval_desc_kernel<EMTK_PATCH_BF16><<<grid, 256, 0, s>>>(t, dimg, job->g0, job->count, job->desc,
+                                                                       job->dest, job->out_stride);
+        else
+            interval_desc_kernel<EMTK_PATCH_F16><<<grid, 256, 0, s>>>(t, dimg, job->g0, job->count, job->desc,
+                                                                      job->dest, job->out_stride);
+        return cudaGetLastError();
     }
     if (most == 0 || t.n == 0) return cudaSuccess;
     int64_t bx = (most + 255) / 256;

@@ -246,3 +246,18 @@ def test_planes_of_odd_unit_counts(emtk, ctx):
     for g, (adc, ntk, thr) in zip(got, planes):
         check_plane(g, adc, ntk, thr)
     assert got[1]["n"] == 0 and got[4]["n"] == 0 and got[3]["n"] > 1000
+
+
+def test_more_planes_than_one_group(emtk, ctx):
+    """70 planes in one call: more than a launch group holds (64), so the
+    call runs two groups; every plane's hits and count must still match."""
+    rng = np.random.default_rng(13)
+    planes = []
+    for i in range(70):
+        nw, nt = 1 + i % 5, 300 + 37 * i
+        ld = (nt + 3) // 4 * 4
+        adc = (rng.standard_normal((nw, ld)) * 3).astype(np.float32)
+        planes.append((adc, nt, 4.0))
+    got = gpu_find(emtk, ctx, planes)
+    for g, (adc, nt, thr) in zip(got, planes):
+        check_plane(g, adc, nt, thr)
