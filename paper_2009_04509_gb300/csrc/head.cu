@@ -127,8 +127,8 @@ __global__ void __launch_bounds__(kThreadsHead) head_kernel(const float *__restr
 // The same tail when a hit has many partial rows (a small launch, whose
 // tiles are split over many CTAs): one warp per hit sums the rows, lane l
 // taking dense-1 outputs 4l .. 4l+3 of every row (512 contiguous bytes per
-// row), and writes bias + ReLU to shared memory; then one thread per hit
-// finishes as above.  HITS hits per block: 8 for small launches (more
+// row), and writes bias + ReLU to shared memory; every thread then computes
+// dense-2 outputs (one per hit and output), and one thread per hit the heads.  HITS hits per block: 8 for small launches (more
 // blocks, so more rows summed at once), 32 above kSmallLaunch hits (fewer
 // blocks loading the dense-2 weights).
 constexpr int kThreadsRows = 256;
@@ -147,6 +147,7 @@ __global__ void __launch_bounds__(kThreadsRows) head_rows_kernel(const float *__
                                                                 const float *__restrict__ mic_b, float *const *dest,
                                                                 int debug_logits) {
     __shared__ float h1s[kHitsRows * kH1Stride];
+    __shared__ float h2s[kHitsRows * (kN2 + 1)];
     __shared__ __align__(16) float w2[kN1][kN2];
     __shared__ __align__(16) float wc[kN2][kNC + 1];
     __shared__ float b2[kN2];
@@ -201,25 +202,21 @@ __global__ void __launch_bounds__(kThreadsRows) head_rows_kernel(const float *__
         o[3] = fmaxf(fmaf(a.w, s1, bb.w), 0.f);
     }
     __syncthreads();
+    // dense-2 with every thread: output j of hit i is thread (32 i + j) mod 256's,
+    // the same fmaf chain over k as head_kernel's
+    for (int o = threadIdx.x; o < kHitsRows * kN2; o += kThreadsRows) {
+        const int i = o / kN2, j = o % kN2;
+        const float *h1 = h1s + i * kH1Stride;
+        float acc = b2[j];
+#pragma unroll 8
+        for (int k = 0; k < kN1; ++k) acc = fmaf(h1[k], w2[k][j], acc);
+        h2s[i * (kN2 + 1) + j] = acc;
+    }
+    __syncthreads();
     if (threadIdx.x >= kHitsRows) return;
     const int64_t h = h0 + threadIdx.x;
     if (h >= n) return;
-    const float *h1 = h1s + threadIdx.x * kH1Stride;
-    float h2[kN2];
-#pragma unroll
-    for (int j = 0; j < kN2; ++j) h2[j] = b2[j];
-    for (int k = 0; k < kN1; ++k) {
-        const float x = h1[k];
-        const float4 *wr = reinterpret_cast<const float4 *>(&w2[k][0]);
-#pragma unroll
-        for (int q = 0; q < kN2 / 4; ++q) {
-            const float4 wv = wr[q];
-            h2[4 * q + 0] = fmaf(x, wv.x, h2[4 * q + 0]);
-            h2[4 * q + 1] = fmaf(x, wv.y, h2[4 * q + 1]);
-            h2[4 * q + 2] = fmaf(x, wv.z, h2[4 * q + 2]);
-            h2[4 * q + 3] = fmaf(x, wv.w, h2[4 * q + 3]);
-        }
-    }
+    const float *h2 = h2s + threadIdx.x * (kN2 + 1);
     float z[kNC + 1] = {cls_b[0], cls_b[1], cls_b[2], mic_b[0]};
 #pragma unroll
     for (int j = 0; j < kN2; ++j) {
