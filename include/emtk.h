@@ -183,6 +183,10 @@ EMTK_API emtk_status emtk_infer_batch(emtk_ctx *ctx, const emtk_request *reqs, i
  * once all of it is enqueued.  Consecutive calls use the two areas in turn,
  * so the copy-in of call i+1 overlaps the kernels of call i (the inference
  * server's input transfer, Sec. 3.3, hidden behind the previous batch).
+ *   - The hit lists are packed on the host into a pinned buffer of the area
+ *     during the call and copied in at once; planes that lie back to back in
+ *     host memory are copied in one piece.  The call waits for the copy-in
+ *     of the area's previous call (two calls back) before packing.
  *   - The host buffers must stay valid and unchanged until `stream` has
  *     completed the call (cudaStreamSynchronize, or an event recorded on
  *     `stream` after the call), and the scores are final only then.

@@ -81,6 +81,7 @@ void free_ctx(emtk_ctx *c) {
     for (auto &st : c->stage) {
         if (st.compute_done) cudaEventSynchronize(st.compute_done);
         if (st.buf) cudaFree(st.buf);
+        if (st.hits_host) cudaFreeHost(st.hits_host);
         if (st.copy_done) cudaEventDestroy(st.copy_done);
         if (st.compute_done) cudaEventDestroy(st.compute_done);
     }
@@ -563,10 +564,14 @@ emtk_status emtk_infer_batch_host(emtk_ctx *c, const emtk_request *reqs, int32_t
         off_adc[i] = need;
         need = up(need + (q.nhits > 0 ? (size_t)q.nwires * (size_t)q.ld * sizeof(float) : 0));
     }
+    // the hit lists back to back (8-byte aligned), so that one copy brings them all
+    const size_t hits0 = need;
     for (int32_t i = 0; i < nreq; ++i) {
         off_hits[i] = need;
-        need = up(need + (size_t)reqs[i].nhits * sizeof(emtk_hit));
+        need += (size_t)reqs[i].nhits * sizeof(emtk_hit);
     }
+    const size_t hit_bytes = need - hits0;
+    need = up(need);
     for (int32_t i = 0; i < nreq; ++i) {
         off_sc[i] = need;
         need = up(need + (size_t)reqs[i].nhits * stride * sizeof(float));
@@ -588,11 +593,28 @@ emtk_status emtk_infer_batch_host(emtk_ctx *c, const emtk_request *reqs, int32_t
         if (e == cudaSuccess) e = cudaMalloc(&st.buf, need);
         if (e == cudaSuccess) st.bytes = need;
     }
+    // the pinned host area for the hit lists: its last copy (two calls back) has landed
+    if (e == cudaSuccess && st.used) e = cudaEventSynchronize(st.copy_done);
+    if (e == cudaSuccess && st.hits_host_bytes < hit_bytes) {
+        if (st.hits_host) e = cudaFreeHost(st.hits_host);
+        st.hits_host = nullptr;
+        st.hits_host_bytes = 0;
+        if (e == cudaSuccess) e = cudaHostAlloc(&st.hits_host, hit_bytes + hit_bytes / 4, cudaHostAllocDefault);
+        if (e == cudaSuccess) st.hits_host_bytes = hit_bytes + hit_bytes / 4;
+    }
     if (e != cudaSuccess) return cuda_status(e);
     char *base = static_cast<char *>(st.buf);
     // copy in on the copy stream, once the area's previous call is done with it
     if (st.used) e = cudaStreamWaitEvent(c->copy_stream, st.compute_done, 0);
     std::vector<emtk_request> dq(reqs, reqs + nreq);
+    // planes: one copy per run of planes contiguous both on the host and in the area
+    const char *run_src = nullptr;
+    size_t run_dst = 0, run_len = 0;
+    auto flush = [&]() {
+        if (run_len > 0 && e == cudaSuccess)
+            e = cudaMemcpyAsync(base + run_dst, run_src, run_len, cudaMemcpyHostToDevice, c->copy_stream);
+        run_len = 0;
+    };
     for (int32_t i = 0; i < nreq && e == cudaSuccess; ++i) {
         const emtk_request &q = reqs[i];
         if (q.nhits == 0) {  // nothing of it is read: no host pointer reaches the batch
@@ -601,15 +623,25 @@ emtk_status emtk_infer_batch_host(emtk_ctx *c, const emtk_request *reqs, int32_t
             dq[i].d_scores = nullptr;
             continue;
         }
-        e = cudaMemcpyAsync(base + off_adc[i], q.d_adc, (size_t)q.nwires * q.ld * sizeof(float),
-                            cudaMemcpyHostToDevice, c->copy_stream);
-        if (e == cudaSuccess)
-            e = cudaMemcpyAsync(base + off_hits[i], q.d_hits, (size_t)q.nhits * sizeof(emtk_hit),
-                                cudaMemcpyHostToDevice, c->copy_stream);
+        const char *src = reinterpret_cast<const char *>(q.d_adc);
+        const size_t len = (size_t)q.nwires * q.ld * sizeof(float);
+        if (run_len > 0 && src == run_src + run_len && off_adc[i] == run_dst + run_len) {
+            run_len += len;
+        } else {
+            flush();
+            run_src = src;
+            run_dst = off_adc[i];
+            run_len = len;
+        }
+        std::memcpy(static_cast<char *>(st.hits_host) + (off_hits[i] - hits0), q.d_hits,
+                    (size_t)q.nhits * sizeof(emtk_hit));
         dq[i].d_adc = reinterpret_cast<const float *>(base + off_adc[i]);
         dq[i].d_hits = reinterpret_cast<const emtk_hit *>(base + off_hits[i]);
         dq[i].d_scores = reinterpret_cast<float *>(base + off_sc[i]);
     }
+    flush();
+    if (e == cudaSuccess && hit_bytes > 0)
+        e = cudaMemcpyAsync(base + hits0, st.hits_host, hit_bytes, cudaMemcpyHostToDevice, c->copy_stream);
     if (e == cudaSuccess) e = cudaEventRecord(st.copy_done, c->copy_stream);
     if (e == cudaSuccess) e = cudaStreamWaitEvent(s, st.copy_done, 0);
     if (e != cudaSuccess) return cuda_status(e);

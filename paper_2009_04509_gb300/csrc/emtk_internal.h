@@ -161,6 +161,8 @@ struct emtk_ctx {
     struct HostStage {
         void *buf = nullptr;
         size_t bytes = 0;
+        void *hits_host = nullptr;  // pinned: the call's hit lists packed, copied in at once
+        size_t hits_host_bytes = 0;
         cudaEvent_t copy_done = nullptr, compute_done = nullptr;
         bool used = false;
     } stage[2];
