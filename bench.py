@@ -584,8 +584,8 @@ def run_sweep(args, rank, world, local_rank):
 HITFIND_THRESHOLD = 15.0  # 5 sigma of the synthetic planes' noise
 # DRAM bytes (read + write) of one hf_find_kernel launch on the full event, from one ncu
 # capture of this workload (profiles/hitfind_full_event.md); null once hitfind.cu changes.
-HF_TRAFFIC_BYTES = 369_189_120 + 4_548_096
-HF_TRAFFIC_SOURCE_SHA256 = "a590b37ebd7512e2"
+HF_TRAFFIC_BYTES = 369_194_496 + 4_427_520
+HF_TRAFFIC_SOURCE_SHA256 = "fb3ec7f9ce385723"
 
 
 def hf_traffic():
