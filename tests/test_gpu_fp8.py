@@ -175,3 +175,23 @@ def test_fp8_full_event_sampled(emtk, ctxs, weights):
         e_all.append(emu)
         r_all.append(ref)
     check_fp8(np.concatenate(g_all), np.concatenate(e_all), np.concatenate(r_all))
+
+
+def test_fp8_largest_sweep_batch(emtk, weights):
+    """65,536 pre-cut patches in one emtk_infer_patches call on a context with
+    default options, as the inference-only sweep runs it; a sample against the
+    emulating oracle and the fp64 one."""
+    n = 65536
+    x = synth.inference_patches(n, seed=0)
+    ctx = emtk.emtk_create(weights, precision="fp8")
+    try:
+        scores = torch.full((n, 4), float("nan"), device="cuda")
+        emtk.emtk_infer_patches(ctx, dev(x), scores)
+        assert emtk.emtk_check(ctx) == emtk.EMTK_OK
+        got = scores.cpu().numpy().astype(np.float64)
+    finally:
+        emtk.emtk_destroy(ctx)
+    assert np.all(np.isfinite(got))
+    idx = np.random.default_rng(22).choice(n, 160, replace=False)
+    ref, emu = references(x[idx], weights)
+    check_fp8(got[idx], emu, ref)

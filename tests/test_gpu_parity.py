@@ -353,3 +353,30 @@ def test_fp32_full_event_sampled(emtk, ctx_factory, weights):
         idx = rng.choice(p.nhits, per, replace=False)
         _, ref = oracle.forward(oracle.extract_patches(p.adc, p.nticks, p.hits[idx]), weights)
         assert np.abs(g[idx, :4] - ref).max() <= TOL_FP32
+
+
+@pytest.mark.parametrize("prec", ["bf16", "fp32"])
+def test_infer_patches_largest_sweep_batch(emtk, weights, prec):
+    """The inference-only sweep's largest batch, 65,536 pre-cut patches in one
+    emtk_infer_patches call on a context with default options, as
+    `bench.py --workload sweep` runs it: every row against the invariants, a
+    sample against the oracle."""
+    n = 65536
+    x = synth.inference_patches(n, seed=0)
+    ctx = emtk.emtk_create(weights, precision=prec)
+    try:
+        scores = torch.full((n, 4), float("nan"), device="cuda")
+        emtk.emtk_infer_patches(ctx, dev(x), scores)
+        assert emtk.emtk_check(ctx) == emtk.EMTK_OK
+        got = scores.cpu().numpy().astype(np.float64)
+    finally:
+        emtk.emtk_destroy(ctx)
+    assert np.all(np.isfinite(got))
+    assert np.all(np.abs(got[:, :3].sum(1) - 1.0) <= 1e-5)
+    idx = np.random.default_rng(21).choice(n, 96, replace=False)
+    _, ref = oracle.forward(x[idx], weights)
+    if prec == "fp32":
+        assert np.abs(got[idx] - ref).max() <= TOL_FP32
+    else:
+        _, emu = oracle.forward(x[idx], weights, emulate="bf16")
+        assert np.abs(got[idx] - emu).max() <= TOL_16
