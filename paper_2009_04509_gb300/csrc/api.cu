@@ -78,6 +78,7 @@ void free_ctx(emtk_ctx *c) {
         cudaStreamDestroy(c->copy_stream);
     }
     if (c->h_totals) cudaFreeHost(c->h_totals);
+    if (c->hf_sums) cudaFree(c->hf_sums);
     for (auto &st : c->stage) {
         if (st.compute_done) cudaEventSynchronize(st.compute_done);
         if (st.buf) cudaFree(st.buf);
@@ -718,11 +719,29 @@ emtk_status emtk_find_hits(emtk_ctx *c, emtk_hitfind_request *reqs, int32_t nreq
             U += nu;
             ++i;
         }
-        cudaError_t e;
+        // the chunk sums: two zeroed halves of hf_sums_cap, grown (and zeroed) when needed
+        cudaError_t e = cudaSuccess;
+        const int64_t nchunks = find_hits_chunks(t, U);
+        if (nchunks > c->hf_sums_cap) {
+            e = cudaStreamSynchronize(s);
+            if (e == cudaSuccess && c->hf_sums) e = cudaFree(c->hf_sums);
+            c->hf_sums = nullptr;
+            c->hf_sums_cap = 0;
+            const int64_t cap = nchunks + nchunks / 4 + 64;
+            if (e == cudaSuccess) e = cudaMalloc(&c->hf_sums, 2 * cap * sizeof(int32_t));
+            if (e == cudaSuccess) e = cudaMemsetAsync(c->hf_sums, 0, 2 * cap * sizeof(int32_t), s);
+            if (e != cudaSuccess) return cuda_status(e);
+            c->hf_sums_cap = cap;
+            c->hf_parity = 0;
+        }
+        int32_t *cur = c->hf_sums + (int64_t)c->hf_parity * c->hf_sums_cap;
+        int32_t *next = c->hf_sums + (int64_t)(1 - c->hf_parity) * c->hf_sums_cap;
         {
             Prof prof(c, EMTK_KERNEL_HITFIND, s);
-            e = launch_find_hits(t, U, scratch, totals, s);
+            e = launch_find_hits(t, U, scratch, cur, next, c->hf_sums_cap, totals, s);
         }
+        if (e == cudaSuccess && U > 0) c->hf_parity ^= 1;
+        if (e != cudaSuccess) c->hf_sums_cap = 0;  // the halves may be dirty: the next call starts afresh
         if (e == cudaSuccess) e = cudaMemcpyAsync(c->h_totals, totals, sizeof(int32_t) * t.n, cudaMemcpyDeviceToHost, s);
         if (e == cudaSuccess) e = cudaStreamSynchronize(s);
         if (e != cudaSuccess) return cuda_status(e);

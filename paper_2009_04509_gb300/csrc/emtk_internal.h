@@ -169,6 +169,11 @@ struct emtk_ctx {
     cudaStream_t copy_stream = nullptr;
     uint64_t host_calls = 0;
     int32_t *h_totals = nullptr;  // pinned: emtk_find_hits' per-plane counts (kMaxHfPlanes)
+    // emtk_find_hits' chunk sums: two halves of hf_sums_cap, used in turn; each
+    // launch clears the other half for the next one
+    int32_t *hf_sums = nullptr;
+    int64_t hf_sums_cap = 0;
+    int hf_parity = 0;
 };
 
 namespace emtk {
@@ -208,11 +213,14 @@ cudaError_t launch_hit_desc(const ReqTable &t, int64_t g0, int32_t count, HitDes
                             int out_stride, cudaStream_t s);
 cudaError_t launch_fill_dest(float *scores, int out_stride, float **dest, int32_t n, cudaStream_t s);
 // Hit finding of the group's planes (hitfind.cu): scratch (256-byte aligned)
-// holds the launch's chunk sums and per-unit run slots; find_hits_unit_cap
-// gives the most units that scratch_bytes holds.  totals[r] receives plane
-// r's hit count.
+// holds per-unit run counts and run slots; find_hits_unit_cap gives the most
+// units that scratch_bytes holds.  The chunk sums live in sums_cur (zero on
+// entry, find_hits_chunks(t, U) of them); the launch zeroes sums_next[0, cap)
+// for the next launch.  totals[r] receives plane r's hit count.
 int64_t find_hits_unit_cap(size_t scratch_bytes);
-cudaError_t launch_find_hits(const HfTable &t, int64_t nunits, void *scratch, int32_t *totals, cudaStream_t s);
+int64_t find_hits_chunks(const HfTable &t, int64_t nunits);
+cudaError_t launch_find_hits(const HfTable &t, int64_t nunits, void *scratch, int32_t *sums_cur, int32_t *sums_next,
+                             int64_t cap, int32_t *totals, cudaStream_t s);
 
 // Network: dense-1 partial sums [splits][n_pad][128] from patches.
 cudaError_t launch_cnn_fp32(const DeviceWeights &w, const float *patches, int32_t n, int splits,

@@ -30,7 +30,8 @@
 //                    threads write consecutive hits.  A unit with more runs
 //                    than slots is scanned again by a warp and written
 //                    directly.  The plane's last unit writes its total.
-// A memset of the chunk sums precedes the two kernels.  The plane is read
+// The chunk sums start at zero: the place kernel of the launch before cleared
+// them (they alternate between two arrays of the context).  The plane is read
 // once from HBM (plus units with more than kRunSlots runs).  No kernel waits
 // on another CTA.  Outputs are ordered by wire, then tick, whatever the
 // launch shape.  The samples are read with the streaming (evict-first) hint:
@@ -50,8 +51,7 @@ constexpr int kHfChunk = 128;   // units per chunk: threads per CTA of the place
 constexpr unsigned kFull = 0xffffffffu;
 static_assert(kSegTicks % (128 * kHfSub) == 0, "a segment is whole load blocks");
 
-// Scratch: the chunk sums (zeroed by the launch, a 256-byte multiple), then
-// per unit its run count and run slots.
+// Scratch: per unit its run count and run slots.
 
 __device__ __forceinline__ int find_plane(const HfTable &t, int64_t u) {
     int r = 0;
@@ -261,7 +261,8 @@ __global__ void __launch_bounds__(kHfChunk) hf_place_kernel(const __grid_constan
                                                              const int32_t *__restrict__ chunk_sum,
                                                              const int32_t *__restrict__ counts,
                                                              const Run *__restrict__ slots,
-                                                             int32_t *__restrict__ total) {
+                                                             int32_t *__restrict__ total,
+                                                             int32_t *__restrict__ sums_next, int64_t cap) {
     constexpr int kWarps = kHfChunk / 32;
     __shared__ int32_t cum[kHfChunk + 1];  // runs copied from the slots before each unit
     __shared__ int32_t out[kHfChunk];      // each unit's offset in its plane
@@ -274,6 +275,9 @@ __global__ void __launch_bounds__(kHfChunk) hf_place_kernel(const __grid_constan
         const int64_t end = tid + 1 < t.n ? t.r[tid + 1].unit0 : nunits;
         if (t.r[tid].unit0 == end) total[tid] = 0;
     }
+    // the next launch's chunk sums start at zero
+    for (int64_t i = (int64_t)blockIdx.x * kHfChunk + tid; i < cap; i += (int64_t)gridDim.x * kHfChunk)
+        sums_next[i] = 0;
     int r = 0;  // the chunk's plane: the last with chunk0 <= blockIdx.x
     while (r + 1 < t.n && t.r[r + 1].chunk0 <= (int64_t)blockIdx.x) ++r;
     const HfDesc &d = t.r[r];
@@ -337,14 +341,20 @@ __global__ void __launch_bounds__(kHfChunk) hf_place_kernel(const __grid_constan
 }  // namespace
 
 int64_t find_hits_unit_cap(size_t scratch_bytes) {
-    // U units use the chunk sums (rounded up to 256 bytes) + U x (count +
-    // slots) bytes; a group has at most U / kHfChunk + kMaxHfPlanes chunks
-    const size_t fixed = 256 + kMaxHfPlanes * sizeof(int32_t);
-    const size_t per_unit = sizeof(int32_t) + kRunSlots * sizeof(Run) + 1;  // + its share of the chunk sums
-    return scratch_bytes > fixed ? (int64_t)((scratch_bytes - fixed) / per_unit) : 0;
+    return (int64_t)(scratch_bytes / (sizeof(int32_t) + kRunSlots * sizeof(Run)));
 }
 
-cudaError_t launch_find_hits(const HfTable &t_in, int64_t nunits, void *scratch, int32_t *totals, cudaStream_t s) {
+int64_t find_hits_chunks(const HfTable &t, int64_t nunits) {
+    int64_t nchunks = 0;
+    for (int r = 0; r < t.n; ++r) {
+        const int64_t nu = (r + 1 < t.n ? t.r[r + 1].unit0 : nunits) - t.r[r].unit0;
+        nchunks += (nu + kHfChunk - 1) / kHfChunk;
+    }
+    return nchunks;
+}
+
+cudaError_t launch_find_hits(const HfTable &t_in, int64_t nunits, void *scratch, int32_t *sums_cur, int32_t *sums_next,
+                             int64_t cap, int32_t *totals, cudaStream_t s) {
     if (nunits <= 0) return cudaMemsetAsync(totals, 0, sizeof(int32_t) * kMaxHfPlanes, s);
     HfTable t = t_in;
     int64_t nchunks = 0;
@@ -353,18 +363,15 @@ cudaError_t launch_find_hits(const HfTable &t_in, int64_t nunits, void *scratch,
         t.r[r].chunk0 = nchunks;
         nchunks += (nu + kHfChunk - 1) / kHfChunk;
     }
-    char *base = static_cast<char *>(scratch);
-    int32_t *chunk_sum = reinterpret_cast<int32_t *>(base);
-    const size_t sums = ((size_t)nchunks * sizeof(int32_t) + 255) & ~(size_t)255;
-    int32_t *counts = reinterpret_cast<int32_t *>(base + sums);
+    if (nchunks > cap) return cudaErrorInvalidValue;
+    int32_t *counts = static_cast<int32_t *>(scratch);
     Run *slots = reinterpret_cast<Run *>(counts + nunits);
-    cudaError_t e = cudaMemsetAsync(chunk_sum, 0, sums, s);
-    if (e != cudaSuccess) return e;
     const unsigned blocks = (unsigned)((nunits + kHfWarps - 1) / kHfWarps);
-    hf_find_kernel<<<blocks, kHfWarps * 32, 0, s>>>(t, nunits, chunk_sum, counts, slots);
-    e = cudaGetLastError();
+    hf_find_kernel<<<blocks, kHfWarps * 32, 0, s>>>(t, nunits, sums_cur, counts, slots);
+    cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    hf_place_kernel<<<(unsigned)nchunks, kHfChunk, 0, s>>>(t, nunits, chunk_sum, counts, slots, totals);
+    hf_place_kernel<<<(unsigned)nchunks, kHfChunk, 0, s>>>(t, nunits, sums_cur, counts, slots, totals, sums_next,
+                                                            cap);
     return cudaGetLastError();
 }
 
