@@ -584,8 +584,8 @@ def run_sweep(args, rank, world, local_rank):
 HITFIND_THRESHOLD = 15.0  # 5 sigma of the synthetic planes' noise
 # DRAM bytes (read + write) of one hf_find_kernel launch on the full event, from one ncu
 # capture of this workload (profiles/hitfind_full_event.md); null once hitfind.cu changes.
-HF_TRAFFIC_BYTES = 369_194_496 + 4_427_520
-HF_TRAFFIC_SOURCE_SHA256 = "fb3ec7f9ce385723"
+HF_TRAFFIC_BYTES = 369_197_824 + 4_327_680
+HF_TRAFFIC_SOURCE_SHA256 = "28b899e456685117"
 
 
 def hf_traffic():
@@ -651,7 +651,7 @@ def run_hitfind(args, rank, world, local_rank):
                       "samples_per_step": samples, "hits_found": nfound,
                       "l2": "flushed between steps (256 MiB write); planes (368.6 MB) exceed L2"},
            "hits_per_s": nfound / (step_ms / 1e3),
-           "roofline": {"bound": "hbm", "kernel": "chunk-sum memset + hf_find_kernel + hf_place_kernel",
+           "roofline": {"bound": "hbm", "kernel": "hf_find_kernel + hf_place_kernel",
                         "achieved": alg_bytes / (kern_ms / 1e3) / 1e9, "peak": peaks["hbm"], "unit": "GB/s",
                         "frac": alg_bytes / (kern_ms / 1e3) / 1e9 / peaks["hbm"],
                         "peak_source": f"{peaks['source']} HBM copy", "algorithmic_bytes": alg_bytes,

@@ -135,7 +135,7 @@ typedef enum {
     EMTK_KERNEL_NETWORK = 2,   /* conv + dense-1 (tensor cores or fp32) */
     EMTK_KERNEL_HEAD = 3,      /* dense-1 sum + dense-2 + heads */
     EMTK_KERNEL_CONVERT = 4,   /* fp32 patches -> 16 bit (emtk_infer_patches) */
-    EMTK_KERNEL_HITFIND = 5,   /* hit finding (emtk_find_hits: chunk-sum memset, find, place) */
+    EMTK_KERNEL_HITFIND = 5,   /* hit finding (emtk_find_hits: find, place) */
     EMTK_NUM_KERNELS = 6
 } emtk_kernel;
 
@@ -288,9 +288,9 @@ typedef struct {
     int32_t reserved;
 } emtk_hitfind_request;
 
-/* Finds the hits of nreq planes (per group of up to 64 planes: a memset of
- * the chunk sums, then two kernels, find and place; each sample is read
- * once, units with more than 128 runs per 2048 ticks twice).  Returns
+/* Finds the hits of nreq planes (per group of up to 64 planes: two kernels,
+ * find and place; each sample is read once, units with more than 128 runs
+ * per 2048 ticks twice).  Returns
  * once the results are complete: it synchronises `stream` to fill each
  * n_found.
  * EMTK_ERR_ARG for negative sizes, ld < nticks, capacity > 0 with a NULL
