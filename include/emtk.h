@@ -221,8 +221,10 @@ EMTK_API emtk_status emtk_extract_patches(emtk_ctx *ctx, const float *d_adc, int
  *     nwires * ((nticks/6 rounded up to a multiple of 8)) * (4 for F32, 2 for
  *     BF16/F16) <= EMTK_STATIC_SCRATCH_BYTES, else EMTK_ERR_ARG and nothing is
  *     enqueued (a 960 x 6000 plane fits in every format).
- *   - The first call on each device looks up the array's device address;
- *     make that first call before any stream capture.
+ *   - The first call on each device looks up the array's device address
+ *     in the device's current context, and so does the first call after
+ *     that context was destroyed and created again (cudaDeviceReset); make
+ *     that first call before any stream capture.
  *   - All calls share the array.  Calls that overlap on the GPU (two streams,
  *     two threads) race; serialise them.  Nothing needs clearing between
  *     calls: every interval a call reads, that call wrote. */
@@ -357,6 +359,31 @@ EMTK_API emtk_status emtk_batcher_stats(emtk_batcher *b, int64_t *batches, int64
  * and frees the batcher's streams and workspaces.  NULL is allowed.  Tickets
  * not yet waited for are dropped. */
 EMTK_API emtk_status emtk_batcher_destroy(emtk_batcher *b);
+
+/* ------------------------------------------------------------------------
+ * Test hooks: host-side fault injection.  They make the failures a service
+ * must survive (an exhausted device, a dispatcher that stops making progress)
+ * happen on the host, with no fault on the GPU.  Not for production use.
+ * -------------------------------------------------------------------- */
+
+/* Arms an allocation failure: `after` more device or pinned-host
+ * allocations of the library succeed, then the next one fails, once, as if
+ * the memory were exhausted (the entry point that made it returns
+ * EMTK_ERR_OOM and frees what it had allocated for that call).  after < 0
+ * disarms.  Process-wide; every allocation of every context counts. */
+EMTK_API void emtk_debug_fail_alloc(int64_t after);
+
+/* Number of device and pinned-host allocations of the library alive now
+ * (weights, workspaces, staging areas, batcher state).  Either pointer may be
+ * NULL. */
+EMTK_API void emtk_debug_alloc_counts(int64_t *device, int64_t *host);
+
+/* stall = 1: the batcher's dispatcher launches nothing until it is called
+ * again with stall = 0 (requests stay queued; emtk_batcher_wait with a
+ * timeout returns EMTK_ERR_TIMEOUT and keeps the ticket).
+ * emtk_batcher_destroy launches what is queued even while stalled.
+ * EMTK_ERR_ARG for a NULL batcher or another value of stall. */
+EMTK_API emtk_status emtk_debug_batcher_stall(emtk_batcher *b, int32_t stall);
 
 #ifdef __cplusplus
 }

@@ -212,9 +212,10 @@ HIT_FIELDS = ("wire", "tick", "start", "end", "peak", "charge")
 
 
 def find_hits(adc, nticks, threshold, lib=None) -> dict:
-    """Hit finding of Sec. 2.1 as read in the design notes: per wire, each
-    maximal run of ticks with adc > threshold is one hit at the run's largest
-    value (earliest on ties).  ``adc`` [nwires][ld] float32, first ``nticks``
+    """Hit finding of Sec. 2.1.  The paper gives no algorithm (only that hits
+    are found on each wire's waveform and carry a time and a charge); the
+    plainest reading: per wire, each maximal run of ticks with adc > threshold
+    is one hit at the run's largest value (earliest on ties).  ``adc`` [nwires][ld] float32, first ``nticks``
     columns are data.  Returns a dict of arrays (wire, tick, start, end: int32;
     peak: float32; charge: float64), ordered by wire then start tick."""
     lib = lib or load()

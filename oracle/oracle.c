@@ -16,8 +16,8 @@
  *             outputs under a softmax and 1 output under a sigmoid.  Dropout
  *             is identity at inference.  11,900,420 parameters in total.
  *
- * Readings where the paper is silent (each one is a choice, listed in the
- * design notes):
+ * Readings where the paper is silent (each one is a choice; the paper fixes
+ * none of them, and another reading would give other patches):
  *   - a time interval is 6 consecutive ticks on a grid fixed to the plane
  *     ([6b, 6b+6)); its value is the fp32 sum a0+a1+...+a5 taken left to
  *     right, then one IEEE fp32 division by 6.  A trailing partial interval
@@ -393,8 +393,9 @@ int or_forward(const or_dims *d, const float *patches, long n,
 
 /* ------------------------------------------------------------- hit finding */
 
-/* Hit finding on the deconvolved waveforms (Sec. 2.1), as read in the
- * design notes.  On each wire w of the plane, a hit is a maximal run of
+/* Hit finding on the deconvolved waveforms (Sec. 2.1).  The paper says only
+ * that hits are found on each wire's deconvolved waveform and carry a time
+ * and a charge; the plainest reading is taken.  On each wire w of the plane, a hit is a maximal run of
  * consecutive ticks t (0 <= t < nticks) with plane[w][t] > threshold
  * (strictly; a NaN is never above).  For each run:
  *   start, end  its first and last tick;

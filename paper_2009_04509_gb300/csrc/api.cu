@@ -1,6 +1,7 @@
 // C ABI of the library (include/emtk.h): argument checks, workspace, the
 // hot-path sequence and counters.  Every launch goes to the caller's stream.
 #include <cuda.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include <algorithm>
 #include <cstdlib>
@@ -45,7 +46,7 @@ constexpr int64_t kPartialCap = 64ll * 1024 * 1024;  // floats of the partial-su
 template <typename T>
 cudaError_t dmalloc(T **p, size_t bytes) {
     void *v = nullptr;
-    cudaError_t e = cudaMalloc(&v, bytes);
+    cudaError_t e = dev_alloc(&v, bytes);
     *p = static_cast<T *>(v);
     return e;
 }
@@ -67,22 +68,22 @@ void free_ctx(emtk_ctx *c) {
         for (void *p : {(void *)w.conv_w, (void *)w.conv_b, (void *)w.fc1_w, (void *)w.fc1_b, (void *)w.fc2_w,
                         (void *)w.fc2_b, (void *)w.cls_w, (void *)w.cls_b, (void *)w.mic_w, (void *)w.mic_b,
                         (void *)w.w1_tiles, (void *)w.convB})
-            if (p) cudaFree(p);
+            dev_free(p);
         delete static_cast<CUtensorMap *>(w.w1_tmap);
     }
     for (void *p : {c->ws.dimg, c->ws.patches, (void *)c->ws.dest, (void *)c->ws.partials, (void *)c->ws.status,
                     (void *)c->ws.hdesc})
-        if (p) cudaFree(p);
+        dev_free(p);
     if (c->copy_stream) {
         cudaStreamSynchronize(c->copy_stream);
         cudaStreamDestroy(c->copy_stream);
     }
-    if (c->h_totals) cudaFreeHost(c->h_totals);
-    if (c->hf_sums) cudaFree(c->hf_sums);
+    host_free(c->h_totals);
+    dev_free(c->hf_sums);
     for (auto &st : c->stage) {
         if (st.compute_done) cudaEventSynchronize(st.compute_done);
-        if (st.buf) cudaFree(st.buf);
-        if (st.hits_host) cudaFreeHost(st.hits_host);
+        dev_free(st.buf);
+        host_free(st.hits_host);
         if (st.copy_done) cudaEventDestroy(st.copy_done);
         if (st.compute_done) cudaEventDestroy(st.compute_done);
     }
@@ -106,13 +107,21 @@ emtk_status check_plane(const float *d_adc, int32_t nwires, int32_t nticks, int6
     return EMTK_OK;
 }
 
-// Profile mode: events around one launch on the caller's stream.
+// Names of the kernel classes in NVTX ranges (a profiler's timeline).
+const char *const kNvtxNames[EMTK_NUM_KERNELS] = {"emtk interval images (patch cut)", "emtk gather / descriptors",
+                                                  "emtk network (conv + dense-1)", "emtk head (dense-2 + heads)",
+                                                  "emtk convert patches", "emtk hit finding"};
+
+// Around one launch: an NVTX range on the host thread (always; free unless a
+// profiler is attached) and, in profile mode, CUDA events on the caller's
+// stream.
 struct Prof {
     emtk_ctx *c;
     int kind;
     cudaStream_t s;
     cudaEvent_t a = nullptr, b = nullptr;
     Prof(emtk_ctx *c_, int kind_, cudaStream_t s_) : c(c_), kind(kind_), s(s_) {
+        nvtxRangePushA(kNvtxNames[kind]);
         c->stats.launches++;
         c->stats.kernel_launches[kind]++;
         if (!c->opt.profile) return;
@@ -124,9 +133,11 @@ struct Prof {
         cudaEventRecord(a, s);
     }
     ~Prof() {
-        if (!a) return;
-        cudaEventRecord(b, s);
-        c->pending.push_back({kind, a, b});
+        if (a) {
+            cudaEventRecord(b, s);
+            c->pending.push_back({kind, a, b});
+        }
+        nvtxRangePop();
     }
 };
 
@@ -155,11 +166,12 @@ emtk_status ensure_dimg(emtk_ctx *c, size_t bytes, cudaStream_t s) {
     // earlier work on this stream may still read the old buffer
     cudaError_t e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return cuda_status(e);
-    if (c->ws.dimg) cudaFree(c->ws.dimg);
+    e = dev_free(c->ws.dimg);
     c->ws.dimg = nullptr;
     c->ws.dimg_bytes = 0;
+    if (e != cudaSuccess) return cuda_status(e);
     const size_t want = bytes + bytes / 4;
-    e = cudaMalloc(&c->ws.dimg, want);
+    e = dev_alloc(&c->ws.dimg, want);
     if (e != cudaSuccess) return cuda_status(e);
     c->ws.dimg_bytes = want;
     return EMTK_OK;
@@ -588,19 +600,19 @@ emtk_status emtk_infer_batch_host(emtk_ctx *c, const emtk_request *reqs, int32_t
     if (e == cudaSuccess && !st.compute_done) e = cudaEventCreateWithFlags(&st.compute_done, cudaEventDisableTiming);
     if (e == cudaSuccess && st.bytes < need) {  // grow: wait for the area's last call, then reallocate
         if (st.used) e = cudaEventSynchronize(st.compute_done);
-        if (e == cudaSuccess && st.buf) e = cudaFree(st.buf);
+        if (e == cudaSuccess) e = dev_free(st.buf);
         st.buf = nullptr;
         st.bytes = 0;
-        if (e == cudaSuccess) e = cudaMalloc(&st.buf, need);
+        if (e == cudaSuccess) e = dev_alloc(&st.buf, need);
         if (e == cudaSuccess) st.bytes = need;
     }
     // the pinned host area for the hit lists: its last copy (two calls back) has landed
     if (e == cudaSuccess && st.used) e = cudaEventSynchronize(st.copy_done);
     if (e == cudaSuccess && st.hits_host_bytes < hit_bytes) {
-        if (st.hits_host) e = cudaFreeHost(st.hits_host);
+        e = host_free(st.hits_host);
         st.hits_host = nullptr;
         st.hits_host_bytes = 0;
-        if (e == cudaSuccess) e = cudaHostAlloc(&st.hits_host, hit_bytes + hit_bytes / 4, cudaHostAllocDefault);
+        if (e == cudaSuccess) e = host_alloc(&st.hits_host, hit_bytes + hit_bytes / 4);
         if (e == cudaSuccess) st.hits_host_bytes = hit_bytes + hit_bytes / 4;
     }
     if (e != cudaSuccess) return cuda_status(e);
@@ -689,10 +701,10 @@ emtk_status emtk_find_hits(emtk_ctx *c, emtk_hitfind_request *reqs, int32_t nreq
     DeviceGuard g(c->device);
     if (!g.ok) return EMTK_ERR_CUDA;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    if (!c->h_totals &&
-        cudaHostAlloc((void **)&c->h_totals, sizeof(int32_t) * kMaxHfPlanes, cudaHostAllocDefault) != cudaSuccess) {
-        c->h_totals = nullptr;
-        return EMTK_ERR_OOM;
+    if (!c->h_totals) {
+        void *h = nullptr;
+        if (host_alloc(&h, sizeof(int32_t) * kMaxHfPlanes) != cudaSuccess) return EMTK_ERR_OOM;
+        c->h_totals = static_cast<int32_t *>(h);
     }
     int32_t *totals = reinterpret_cast<int32_t *>(c->ws.partials);
     void *scratch = reinterpret_cast<char *>(c->ws.partials) + 256;
@@ -724,11 +736,11 @@ emtk_status emtk_find_hits(emtk_ctx *c, emtk_hitfind_request *reqs, int32_t nreq
         const int64_t nchunks = find_hits_chunks(t, U);
         if (nchunks > c->hf_sums_cap) {
             e = cudaStreamSynchronize(s);
-            if (e == cudaSuccess && c->hf_sums) e = cudaFree(c->hf_sums);
+            if (e == cudaSuccess) e = dev_free(c->hf_sums);
             c->hf_sums = nullptr;
             c->hf_sums_cap = 0;
             const int64_t cap = nchunks + nchunks / 4 + 64;
-            if (e == cudaSuccess) e = cudaMalloc(&c->hf_sums, 2 * cap * sizeof(int32_t));
+            if (e == cudaSuccess) e = dmalloc(&c->hf_sums, 2 * cap * sizeof(int32_t));
             if (e == cudaSuccess) e = cudaMemsetAsync(c->hf_sums, 0, 2 * cap * sizeof(int32_t), s);
             if (e != cudaSuccess) return cuda_status(e);
             c->hf_sums_cap = cap;
@@ -741,10 +753,14 @@ emtk_status emtk_find_hits(emtk_ctx *c, emtk_hitfind_request *reqs, int32_t nreq
             e = launch_find_hits(t, U, scratch, cur, next, c->hf_sums_cap, totals, s);
         }
         if (e == cudaSuccess && U > 0) c->hf_parity ^= 1;
-        if (e != cudaSuccess) c->hf_sums_cap = 0;  // the halves may be dirty: the next call starts afresh
         if (e == cudaSuccess) e = cudaMemcpyAsync(c->h_totals, totals, sizeof(int32_t) * t.n, cudaMemcpyDeviceToHost, s);
         if (e == cudaSuccess) e = cudaStreamSynchronize(s);
-        if (e != cudaSuccess) return cuda_status(e);
+        if (e != cudaSuccess) {
+            // the launch or the kernels may have stopped before the place kernel cleared
+            // the other half: the next call reallocates and zeroes both halves
+            c->hf_sums_cap = 0;
+            return cuda_status(e);
+        }
         for (int r = 0; r < t.n; ++r) reqs[first + r].n_found = c->h_totals[r];
     }
     return EMTK_OK;

@@ -71,6 +71,7 @@ struct emtk_batcher {
     uint64_t seq = 0;
     bool stop = false;
     bool dispatch_done = false;
+    bool stalled = false;  // test knob (emtk_debug_batcher_stall): the dispatcher launches nothing
     int64_t n_batches = 0, n_requests = 0, n_hits = 0;
 
     std::thread dispatcher, completer;
@@ -84,6 +85,10 @@ void dispatch_loop(emtk_batcher *b) {
     for (;;) {
         if (b->queue.empty()) {
             if (b->stop) break;
+            b->cv_dispatch.wait(lk);
+            continue;
+        }
+        if (b->stalled && !b->stop) {  // a stalled dispatcher, until released or destroyed
             b->cv_dispatch.wait(lk);
             continue;
         }
@@ -175,7 +180,7 @@ void free_batcher(emtk_batcher *b) {
         }
         emtk::destroy_lane_ctx(l.ctx);
     }
-    if (b->h_status) cudaFreeHost(b->h_status);
+    emtk::host_free(b->h_status);
     delete b;
 }
 
@@ -196,9 +201,13 @@ emtk_status emtk_batcher_create(emtk_ctx *ctx, int32_t nstreams, int32_t max_hit
     int prev = -1;
     if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
     emtk_status st = cudaSetDevice(b->device) == cudaSuccess ? EMTK_OK : EMTK_ERR_CUDA;
-    if (st == EMTK_OK && cudaHostAlloc((void **)&b->h_status, kMaxInflight * sizeof(int), cudaHostAllocDefault) !=
-                             cudaSuccess)
-        st = EMTK_ERR_OOM;
+    if (st == EMTK_OK) {
+        void *h = nullptr;
+        if (emtk::host_alloc(&h, kMaxInflight * sizeof(int)) != cudaSuccess)
+            st = EMTK_ERR_OOM;
+        else
+            b->h_status = static_cast<int *>(h);
+    }
     for (int i = 0; st == EMTK_OK && i < kMaxInflight; ++i) {
         cudaEvent_t ev;
         if (cudaEventCreateWithFlags(&ev, cudaEventDisableTiming) != cudaSuccess)
@@ -275,6 +284,16 @@ emtk_status emtk_batcher_stats(emtk_batcher *b, int64_t *batches, int64_t *reque
     if (batches) *batches = b->n_batches;
     if (requests) *requests = b->n_requests;
     if (hits) *hits = b->n_hits;
+    return EMTK_OK;
+}
+
+emtk_status emtk_debug_batcher_stall(emtk_batcher *b, int32_t stall) {
+    if (!b || (stall != 0 && stall != 1)) return EMTK_ERR_ARG;
+    {
+        std::lock_guard<std::mutex> lk(b->mu);
+        b->stalled = stall != 0;
+    }
+    b->cv_dispatch.notify_all();
     return EMTK_OK;
 }
 

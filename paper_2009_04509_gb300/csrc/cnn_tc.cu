@@ -854,12 +854,14 @@ cudaError_t prepare_tc_weights(DeviceWeights &w, const emtk_weights &hw, TcMode 
         }
     }
     const size_t w1_bytes = f8 ? nw1 : nw1 * 2;
-    cudaError_t e = cudaMalloc(&w.w1_tiles, w1_bytes);
+    cudaError_t e = dev_alloc(&w.w1_tiles, w1_bytes);
     if (e != cudaSuccess) return e;
     e = cudaMemcpy(w.w1_tiles, f8 ? (const void *)tiles8.data() : (const void *)tiles.data(), w1_bytes,
                    cudaMemcpyHostToDevice);
     if (e != cudaSuccess) return e;
-    e = cudaMalloc(&w.convB, cb.size() * 2);
+    void *cbp = nullptr;
+    e = dev_alloc(&cbp, cb.size() * 2);
+    w.convB = static_cast<uint16_t *>(cbp);
     if (e != cudaSuccess) return e;
     e = cudaMemcpy(w.convB, cb.data(), cb.size() * 2, cudaMemcpyHostToDevice);
     if (e != cudaSuccess) return e;

@@ -178,6 +178,14 @@ struct emtk_ctx {
 
 namespace emtk {
 
+// ---- allocations (alloc.cu): every device and pinned-host allocation of the
+// library, counted; emtk_debug_fail_alloc can make one of them fail.  *p is
+// null after a failure; freeing null is a no-op.
+cudaError_t dev_alloc(void **p, size_t bytes);
+cudaError_t dev_free(void *p);
+cudaError_t host_alloc(void **p, size_t bytes);
+cudaError_t host_free(void *p);
+
 // ---- host helpers shared by the API and the request batcher (api.cu)
 // The checks emtk_infer_batch applies to one request.
 emtk_status validate_request(const emtk_request &q);

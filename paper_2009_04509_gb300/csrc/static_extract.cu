@@ -16,6 +16,9 @@
 // between calls.  All calls share the one array: calls that overlap on the
 // GPU (on two streams, or two host threads) race and must be serialised by
 // the caller.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
 #include <mutex>
 
 #include "emtk_internal.h"
@@ -28,21 +31,60 @@ constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) unsigned char g_interval_scratch[kStaticScratchBytes];
 
+// The array's device address belongs to the device's context: a context that
+// is destroyed and created again (cudaDeviceReset, a framework resetting the
+// device) may load the library's module at another address.  So the address
+// is kept together with the unique id of the context it was looked up in,
+// and looked up again when the current context is another one.
+struct ScratchSlot {
+    unsigned long long ctx_id;
+    void *addr;
+};
 std::mutex g_scratch_mutex;
-void *g_scratch_addr[kMaxDevices];  // device address of g_interval_scratch, per device
+ScratchSlot g_scratch_slot[kMaxDevices];
+PFN_cuCtxGetCurrent_v4000 g_ctx_get_current = nullptr;
+PFN_cuCtxGetId_v12000 g_ctx_get_id = nullptr;
 
-// Looks up the array's device address once per device, with that device
-// current.  In host code the name g_interval_scratch is only a host-side
-// stand-in, never a device address.
+// Resolves the two driver calls once (through the runtime, so the library
+// needs no link against the driver library).
+bool resolve_driver_calls() {
+    if (g_ctx_get_current && g_ctx_get_id) return true;
+    void *a = nullptr, *b = nullptr;
+    cudaDriverEntryPointQueryResult qa, qb;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &a, 4000, cudaEnableDefault, &qa) != cudaSuccess ||
+        cudaGetDriverEntryPointByVersion("cuCtxGetId", &b, 12000, cudaEnableDefault, &qb) != cudaSuccess ||
+        qa != cudaDriverEntryPointSuccess || qb != cudaDriverEntryPointSuccess || !a || !b)
+        return false;
+    g_ctx_get_current = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(a);
+    g_ctx_get_id = reinterpret_cast<PFN_cuCtxGetId_v12000>(b);
+    return true;
+}
+
+// The array's device address in the current context of `device` (the
+// caller's current device).  Looked up with cudaGetSymbolAddress the first
+// time a context is seen; in host code the name g_interval_scratch is only a
+// host-side stand-in, never a device address.
 cudaError_t scratch_address(int device, void **out) {
     std::lock_guard<std::mutex> lock(g_scratch_mutex);
-    if (g_scratch_addr[device] == nullptr) {
+    if (!resolve_driver_calls()) return cudaErrorNotSupported;
+    CUcontext ctx = nullptr;
+    if (g_ctx_get_current(&ctx) != CUDA_SUCCESS) return cudaErrorInitializationError;
+    if (ctx == nullptr) {  // no context bound to this thread yet: bind the device's primary one
+        const cudaError_t e = cudaSetDevice(device);
+        if (e != cudaSuccess) return e;
+        if (g_ctx_get_current(&ctx) != CUDA_SUCCESS || ctx == nullptr) return cudaErrorInitializationError;
+    }
+    unsigned long long id = 0;
+    if (g_ctx_get_id(ctx, &id) != CUDA_SUCCESS) return cudaErrorInitializationError;
+    ScratchSlot &slot = g_scratch_slot[device];
+    if (slot.addr == nullptr || slot.ctx_id != id) {
         void *p = nullptr;
         const cudaError_t e = cudaGetSymbolAddress(&p, g_interval_scratch);
         if (e != cudaSuccess) return e;
-        g_scratch_addr[device] = p;
+        slot.addr = p;
+        slot.ctx_id = id;
     }
-    *out = g_scratch_addr[device];
+    *out = slot.addr;
     return cudaSuccess;
 }
 

@@ -26,7 +26,8 @@ EXPORTED = ("emtk_default_options", "emtk_create", "emtk_destroy", "emtk_infer",
             "emtk_extract_patches", "emtk_infer_patches", "emtk_check", "emtk_get_stats",
             "emtk_status_string", "emtk_extract_patches_static", "emtk_batcher_create", "emtk_batcher_submit",
             "emtk_batcher_wait", "emtk_batcher_stats", "emtk_batcher_destroy", "emtk_get_fp8_scales",
-            "emtk_find_hits", "emtk_infer_batch_host")
+            "emtk_find_hits", "emtk_infer_batch_host", "emtk_debug_fail_alloc", "emtk_debug_alloc_counts",
+            "emtk_debug_batcher_stall")
 EMTK_STATIC_SCRATCH_BYTES = 4 << 20
 
 _vp = ctypes.c_void_p
@@ -107,6 +108,12 @@ def load_library(path: str | None = None):
     lib.emtk_infer_batch_host.argtypes = [_vp, ctypes.POINTER(emtk_request), ctypes.c_int32, _vp]
     lib.emtk_infer_batch_host.restype = ctypes.c_int
     lib.emtk_find_hits.restype = ctypes.c_int
+    lib.emtk_debug_fail_alloc.argtypes = [ctypes.c_int64]
+    lib.emtk_debug_fail_alloc.restype = None
+    lib.emtk_debug_alloc_counts.argtypes = [ctypes.POINTER(ctypes.c_int64), ctypes.POINTER(ctypes.c_int64)]
+    lib.emtk_debug_alloc_counts.restype = None
+    lib.emtk_debug_batcher_stall.argtypes = [_vp, ctypes.c_int32]
+    lib.emtk_debug_batcher_stall.restype = ctypes.c_int
     for name in ("emtk_batcher_create", "emtk_batcher_submit", "emtk_batcher_wait", "emtk_batcher_stats",
                  "emtk_batcher_destroy"):
         getattr(lib, name).restype = ctypes.c_int
@@ -313,3 +320,20 @@ def emtk_batcher_stats(b) -> dict:
 
 def emtk_batcher_destroy(b) -> None:
     _check(load_library().emtk_batcher_destroy(b), "emtk_batcher_destroy")
+
+
+# ------------------------------------------------------------- test hooks
+def emtk_debug_fail_alloc(after: int) -> None:
+    """The allocation after ``after`` more successful ones fails, once (< 0 disarms)."""
+    load_library().emtk_debug_fail_alloc(int(after))
+
+
+def emtk_debug_alloc_counts() -> tuple:
+    """(device, pinned host) allocations of the library alive now."""
+    d, h = ctypes.c_int64(), ctypes.c_int64()
+    load_library().emtk_debug_alloc_counts(ctypes.byref(d), ctypes.byref(h))
+    return d.value, h.value
+
+
+def emtk_debug_batcher_stall(b, stall: bool) -> None:
+    _check(load_library().emtk_debug_batcher_stall(b, int(bool(stall))), "emtk_debug_batcher_stall")

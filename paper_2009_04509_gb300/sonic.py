@@ -85,7 +85,9 @@ def paper_job(dynamic_batching: bool = True, link_gbps: float = 2.0, large_batch
 def gb300_job(hits_per_s: float, inferences: int = PAPER_INFERENCES, t_cpu: float = PAPER_T_CPU,
               p: float = PAPER_P) -> Job:
     """The paper's CPU job with its offloaded part replaced by this library's
-    measured throughput: the patch cut now runs on the GPU (no CPU
-    preprocessing) and, in one process, there is no network transfer or round
-    trip; the host-device copies are inside the end-to-end throughput."""
+    measured throughput.  ``hits_per_s`` must be an end-to-end figure, taken
+    through the call with host buffers (the planes and hits copied to the
+    device, the scores copied back), so that the host-device copies are
+    inside t_gpu; the patch cut runs on the GPU (no CPU preprocessing) and, in
+    one process, there is no network transfer or round trip."""
     return Job(t_cpu=t_cpu, p=p, t_gpu=inferences / hits_per_s)

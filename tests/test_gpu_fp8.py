@@ -34,7 +34,6 @@ ARGMAX_EMU = 0.995
 ARGMAX_FP64 = 0.95
 TOL_FP64_UNSAT = 5e-2
 S_A = 2.0 ** -4
-SAMPLE = 256
 
 
 @pytest.fixture(scope="module")
@@ -151,32 +150,6 @@ def test_fp8_infer_patches_lognormal(emtk, ctxs, weights):
     check_fp8(scores.cpu().numpy().astype(np.float64), emu, ref)
 
 
-def test_fp8_full_event_sampled(emtk, ctxs, weights):
-    """The full 18-plane event (60,000 hits) in one batched call, the
-    benchmark's launch; a sample of hits against the oracle."""
-    planes = synth.full_event(seed=0)
-    ctx = ctxs["a"]
-    items, outs = [], []
-    for p in planes:
-        s = torch.full((p.nhits, 8), float("nan"), device="cuda")
-        items.append((dev(p.adc), p.nticks, dev(p.hits), s))
-        outs.append(s)
-    emtk.emtk_infer_batch(ctx, items)
-    assert emtk.emtk_check(ctx) == emtk.EMTK_OK
-    got = [s.cpu().numpy().astype(np.float64) for s in outs]
-    assert np.all(np.isfinite(np.concatenate(got)[:, :4]))
-    rng = np.random.default_rng(11)
-    per = SAMPLE // len(planes) + 1
-    g_all, e_all, r_all = [], [], []
-    for p, g in zip(planes, got):
-        idx = rng.choice(p.nhits, per, replace=False)
-        ref, emu = references(oracle.extract_patches(p.adc, p.nticks, p.hits[idx]), weights)
-        g_all.append(g[idx])
-        e_all.append(emu)
-        r_all.append(ref)
-    check_fp8(np.concatenate(g_all), np.concatenate(e_all), np.concatenate(r_all))
-
-
 def test_fp8_largest_sweep_batch(emtk, weights):
     """65,536 pre-cut patches in one emtk_infer_patches call on a context with
     default options, as the inference-only sweep runs it; a sample against the
@@ -192,6 +165,6 @@ def test_fp8_largest_sweep_batch(emtk, weights):
     finally:
         emtk.emtk_destroy(ctx)
     assert np.all(np.isfinite(got))
-    idx = np.random.default_rng(22).choice(n, 160, replace=False)
+    idx = np.random.default_rng(22).choice(n, 2048, replace=False)
     ref, emu = references(x[idx], weights)
     check_fp8(got[idx], emu, ref)

@@ -12,6 +12,7 @@ import ctypes
 import numpy as np
 import pytest
 
+import oracle
 from paper_2009_04509_gb300 import synth
 
 torch = pytest.importorskip("torch")
@@ -24,6 +25,7 @@ def emtk():
         pytest.skip("no CUDA device")
     from paper_2009_04509_gb300 import build, emtk as m
     build.build()
+    oracle.build()
     return m
 
 
@@ -37,25 +39,48 @@ def _static_call(m, adc, nticks, hits, out, fmt):
         ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
 
 
+def _want(plane, fmt):
+    """The oracle's patch cut, in the output format (16-bit: round to nearest even)."""
+    p = oracle.extract_patches(plane.adc, plane.nticks, plane.hits)
+    return p.view(np.uint32) if fmt == "f32" else oracle.round_bf16(p)
+
+
 @pytest.mark.parametrize("fmt", ["f32", "bf16"])
 def test_static_patch_cut_matches_context_call(emtk, fmt):
     """Two calls in a row (a full-size 960-wire plane, then a smaller ragged
-    one) give the same patches as the existing context-based entry point."""
+    one) give the oracle's patches bit for bit, and the same patches as the
+    existing context-based entry point; the device's free memory does not
+    change across the calls."""
     dev = torch.device("cuda:0")
     big = synth.full_event(seed=3, n_apa=1)[2]                 # 960 x 6000
     small = synth.single_plane(seed=4, nwires=37, nhits=300, nticks=1996)   # 1996 % 6 != 0
     ctx = emtk.emtk_create(synth.he_normal_weights(0), precision="bf16")
     try:
+        bufs = []
         for plane in (big, small):
             adc = torch.from_numpy(plane.adc).to(dev)
             hits = torch.from_numpy(plane.hits).to(dev)
             dt = torch.float32 if fmt == "f32" else torch.int16
             got = torch.full((plane.nhits, 48, 48), -1, dtype=dt, device=dev)
             want = torch.zeros((plane.nhits, 48, 48), dtype=dt, device=dev)
+            bufs.append((plane, adc, hits, got, want))
+        # a first call loads the library's module holding the fixed array (the CUDA
+        # runtime loads modules lazily) and looks up the array's address; it is
+        # the calls after it that must leave the device's free memory unchanged
+        plane, adc, hits, got, _ = bufs[1]
+        assert _static_call(emtk, adc, plane.nticks, hits, got, fmt) == emtk.EMTK_OK
+        torch.cuda.synchronize()
+        free0 = torch.cuda.mem_get_info()[0]
+        for plane, adc, hits, got, _ in bufs:
             assert _static_call(emtk, adc, plane.nticks, hits, got, fmt) == emtk.EMTK_OK
+        torch.cuda.synchronize()
+        assert torch.cuda.mem_get_info()[0] == free0    # nothing was allocated on the device
+        for plane, adc, hits, got, want in bufs:
             emtk.emtk_extract_patches(ctx, adc, plane.nticks, hits, want, fmt)
             torch.cuda.synchronize()
             assert torch.equal(got, want)      # the patch cut is exact: tolerance zero
+            g = got.cpu().numpy()
+            assert np.array_equal(g.view(np.uint32) if fmt == "f32" else g.view(np.uint16), _want(plane, fmt))
     finally:
         emtk.emtk_destroy(ctx)
 
