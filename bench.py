@@ -245,7 +245,7 @@ def main():
     ap.add_argument("--clients", type=int, default=64, help="service workload: client threads (one event each)")
     ap.add_argument("--streams", type=int, default=8, help="service workload: batcher streams")
     ap.add_argument("--max-delay-us", type=int, default=500, help="service workload: batcher delay")
-    ap.add_argument("--precision", default="bf16", choices=["bf16", "fp16", "fp8", "fp32"])
+    ap.add_argument("--precision", default="bf16", choices=["bf16", "fp16", "fp8", "fp32", "tf32"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     args = ap.parse_args()
@@ -341,6 +341,8 @@ def main():
     union = window_union_bytes(planes)
     if args.precision == "fp32":  # the fp32 path writes every patch
         patch_bytes = nhits * 48 * 48 * 4
+    elif args.precision == "tf32":  # the split path writes 4-byte interval words
+        patch_bytes = sum(p.nwires * (p.nticks // 6) for p in planes) * 4
     else:  # the 16-bit paths write the interval image; the network reads the windows from it
         patch_bytes = sum(p.nwires * (p.nticks // 6) for p in planes) * 2
     cut_ms = (kms["intervals"] + kms["gather"]) / args.steps
@@ -370,8 +372,10 @@ def main():
                                                                     if args.workload == "full_event" else ""),
                    "parallelism": f"replicas x{world} (independent events, no collective)"},
         "gpu_launches": launches,
-        "roofline": {"bound": "alu" if args.precision == "fp32" else "tensor", "kernel": "cnn_tc_kernel (conv 5x5x48 + dense-1, tcgen05)"
-                     if args.precision != "fp32" else "cnn_fp32_kernel",
+        "roofline": {"bound": "alu" if args.precision == "fp32" else "tensor",
+                     "kernel": {"fp32": "cnn_fp32_kernel",
+                                "tf32": "cnn_split_kernel (conv 5x5x48 + dense-1, tcgen05, split fp16 operands)"}.get(
+                         args.precision, "cnn_tc_kernel (conv 5x5x48 + dense-1, tcgen05)"),
                      "achieved": achieved, "peak": net_peak, "unit": "TFLOP/s",
                      "frac": achieved / net_peak,
                      "peak_source": net_peak_src, "frac_of_sustained": None if args.precision == "fp32"

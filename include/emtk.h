@@ -69,7 +69,22 @@ typedef enum {
  *              max|W1| * s_w <= 448; the fp32 sums are multiplied by
  *              1 / (s_a s_w) before the dense-1 bias (emtk_get_fp8_scales).
  *              Patches are bf16.
- *   EMTK_TF32: reserved; emtk_create returns EMTK_ERR_UNSUPPORTED. */
+ *   EMTK_TF32: fp32 accuracy on the tcgen05 tensor cores.  Every fp32
+ *              operand of the conv and of dense-1 (patch pixels, conv
+ *              weights and bias, conv activations, dense-1 weights) is
+ *              written as the sum of two fp16 values, a head and a tail
+ *              (22 significant bits together, as many as a TF32 head and
+ *              tail), and every product is taken as three fp16 products
+ *              (head x head, head x tail, tail x head) accumulated in fp32:
+ *              the operand-splitting method of Markidis et al. (2018), at
+ *              the fp16 tensor rate, which is twice that of the TF32 format.
+ *              Power-of-two scales keep heads and tails inside fp16's range:
+ *              pixels by 2^-4, activations by 2^-4, dense-1 weights by the
+ *              largest 2^k with max|W1| 2^k <= 2^14, conv weights and bias
+ *              (times 2^-4) by the largest 2^k with their largest magnitude
+ *              times 2^k <= 2^14.  Interval values and conv activations must
+ *              stay below 2^20 in magnitude; beyond that the scores are
+ *              undefined. */
 typedef enum { EMTK_FP32 = 0, EMTK_TF32 = 1, EMTK_BF16 = 2, EMTK_FP16 = 3, EMTK_FP8 = 4 } emtk_precision;
 
 /* Element type of a patch buffer. */
@@ -152,9 +167,9 @@ typedef struct {
 EMTK_API void emtk_default_options(emtk_options *out);
 
 /* Creates a context on CUDA device `device`: uploads and converts the
- * weights and allocates the workspace.  Returns EMTK_ERR_UNSUPPORTED for
- * EMTK_TF32 or a device older than compute capability 10.3 when a
- * tensor-core precision is asked for.  *out is NULL on failure. */
+ * weights and allocates the workspace.  Returns EMTK_ERR_UNSUPPORTED on a
+ * device other than compute capability 10.3 (the library is built for
+ * sm_103a only).  *out is NULL on failure. */
 EMTK_API emtk_status emtk_create(const emtk_weights *w, const emtk_options *opt, int device, emtk_ctx **out);
 
 /* Frees the context (synchronises its device first).  NULL is accepted. */

@@ -26,16 +26,24 @@ struct DeviceGuard {  // restores the caller's current device
     }
 };
 
-bool tensor_precision(emtk_precision p) { return p == EMTK_BF16 || p == EMTK_FP16 || p == EMTK_FP8; }
-
-TcMode tc_mode(emtk_precision p) { return p == EMTK_FP16 ? kTcFp16 : p == EMTK_FP8 ? kTcFp8 : kTcBf16; }
-
-// EMTK_FP8 keeps the conv in bf16, so its patches are bf16
-emtk_patch_format patch_format(emtk_precision p) {
-    return (p == EMTK_BF16 || p == EMTK_FP8) ? EMTK_PATCH_BF16 : p == EMTK_FP16 ? EMTK_PATCH_F16 : EMTK_PATCH_F32;
+bool tensor_precision(emtk_precision p) {
+    return p == EMTK_BF16 || p == EMTK_FP16 || p == EMTK_FP8 || p == EMTK_TF32;
 }
 
-size_t patch_elem_bytes(emtk_patch_format f) { return f == EMTK_PATCH_F32 ? 4 : 2; }
+TcMode tc_mode(emtk_precision p) {
+    return p == EMTK_FP16 ? kTcFp16 : p == EMTK_FP8 ? kTcFp8 : p == EMTK_TF32 ? kTcSplit : kTcBf16;
+}
+
+// EMTK_FP8 keeps the conv in bf16, so its patches are bf16; EMTK_TF32 uses
+// fp16 head + tail words
+emtk_patch_format patch_format(emtk_precision p) {
+    return (p == EMTK_BF16 || p == EMTK_FP8) ? EMTK_PATCH_BF16
+           : p == EMTK_FP16                  ? EMTK_PATCH_F16
+           : p == EMTK_TF32                  ? kPatchSplit16
+                                             : EMTK_PATCH_F32;
+}
+
+size_t patch_elem_bytes(emtk_patch_format f) { return (f == EMTK_PATCH_F32 || f == kPatchSplit16) ? 4 : 2; }
 
 int out_stride(const emtk_ctx *c) { return c->opt.debug_logits ? 8 : 4; }
 
@@ -69,7 +77,7 @@ void free_ctx(emtk_ctx *c) {
                         (void *)w.fc2_b, (void *)w.cls_w, (void *)w.cls_b, (void *)w.mic_w, (void *)w.mic_b,
                         (void *)w.w1_tiles, (void *)w.convB})
             dev_free(p);
-        delete static_cast<CUtensorMap *>(w.w1_tmap);
+        delete[] static_cast<CUtensorMap *>(w.w1_tmap);
     }
     for (void *p : {c->ws.dimg, c->ws.patches, (void *)c->ws.dest, (void *)c->ws.partials, (void *)c->ws.status,
                     (void *)c->ws.hdesc})
@@ -396,8 +404,6 @@ emtk_status emtk_create(const emtk_weights *w, const emtk_options *opt, int devi
     if (o.max_hits <= 0 || o.wait_timeout_ns <= 0 || (o.debug_logits != 0 && o.debug_logits != 1) ||
         (o.profile != 0 && o.profile != 1) || (o.debug_stall != 0 && o.debug_stall != 1))
         return EMTK_ERR_ARG;
-    if (o.precision == EMTK_TF32) return EMTK_ERR_UNSUPPORTED;
-
     int ndev = 0;
     if (cudaGetDeviceCount(&ndev) != cudaSuccess || device >= ndev) return EMTK_ERR_CUDA;
     DeviceGuard g(device);
@@ -426,7 +432,10 @@ emtk_status emtk_create(const emtk_weights *w, const emtk_options *opt, int devi
     if (e == cudaSuccess) e = upload(&d.mic_w, w->mic_w, kN2);
     if (e == cudaSuccess) e = upload(&d.mic_b, w->mic_b, 1);
     if (e == cudaSuccess) {
-        if (tensor_precision(o.precision)) {
+        if (o.precision == EMTK_TF32) {
+            e = prepare_split_weights(d, *w);
+            if (e == cudaSuccess) e = init_split_kernel_attrs();
+        } else if (tensor_precision(o.precision)) {
             e = prepare_tc_weights(d, *w, tc_mode(o.precision));
             if (e == cudaSuccess) e = init_tc_kernel_attrs();
         } else {

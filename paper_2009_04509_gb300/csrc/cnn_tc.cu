@@ -36,6 +36,7 @@
 #include <vector>
 
 #include "emtk_internal.h"
+#include "tc_ptx.cuh"
 
 namespace emtk {
 namespace {
@@ -102,204 +103,6 @@ constexpr int kSmemBytesTC = kSmemUsed + 1024;  // slack for 1024-byte alignment
 static_assert(kSmemBytesTC <= 232448, "shared memory budget");
 static_assert(kSlotCol0 + kSlots * kSlotCols <= kTmemCols, "TMEM budget");
 static_assert(kQ % kPosPerW1 == 0, "quads do not straddle rows");
-
-// ------------------------------------------------------------ PTX helpers
-__device__ __forceinline__ uint32_t smem_u32(const void *p) {
-    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
-}
-// The thread may be suspended until the phase completes, for at most
-// kSuspendHintNs per call (a hint: the callers' loops bound the total wait);
-// a suspended waiter takes no issue slots from its sub-partition's warps.
-constexpr uint32_t kSuspendHintNs = 100000;
-__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(bar), "r"(parity), "n"(kSuspendHintNs)
-        : "memory");
-    return ok != 0;
-}
-__device__ __forceinline__ uint64_t global_timer_ns() {
-    uint64_t t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    return t;
-}
-
-struct Guard {
-    volatile uint32_t *abort;
-    int *status;
-    int64_t timeout_ns;
-};
-
-// Waits for the phase of `parity` to complete.  Gives up (false) when the
-// CTA's abort flag is raised or after timeout_ns, raising the flag and the
-// status bit itself in the second case.
-__device__ __noinline__ bool wait_slow(uint32_t bar, uint32_t parity, Guard g) {
-    const uint64_t t0 = global_timer_ns();
-    for (uint32_t i = 1;; ++i) {
-        if (mbar_try_wait(bar, parity)) return true;
-        if ((i & 31u) == 0) {
-            if (*g.abort) return false;
-            if ((int64_t)(global_timer_ns() - t0) > g.timeout_ns) {
-                *g.abort = 1u;
-                atomicOr(g.status, 1);
-                return false;
-            }
-        }
-    }
-}
-
-__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, const Guard &g) {
-    if (mbar_try_wait(bar, parity)) return true;
-    return wait_slow(bar, parity, g);
-}
-
-// Lane 0 waits; the outcome is broadcast so the whole warp takes the same path.
-__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, Guard g, int lane) {
-    int ok = 1;
-    if (lane == 0) ok = wait_bounded(bar, parity, g) ? 1 : 0;
-    ok = __shfl_sync(0xffffffffu, ok, 0);
-    __syncwarp();
-    return ok != 0;
-}
-
-__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int c0, int c1,
-                                            int c2) {
-    asm volatile(
-        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4, %5}], "
-        "[%2];" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "r"(c2)
-        : "memory");
-}
-
-__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
-__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
-
-// D[tmem] (+)= A[tmem] * B[smem desc], kind::f16, one CTA.
-__device__ __forceinline__ void mma_ts(uint32_t d, uint32_t a, uint64_t bdesc, uint32_t idesc, uint32_t accum) {
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d),
-        "r"(a), "l"(bdesc), "r"(idesc), "r"(accum)
-        : "memory");
-}
-// D[tmem] (+)= A[smem desc] * B[smem desc], kind::f16, one CTA.
-__device__ __forceinline__ void mma_ss(uint32_t d, uint64_t adesc, uint64_t bdesc, uint32_t idesc, uint32_t accum) {
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d),
-        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accum)
-        : "memory");
-}
-// D[tmem] (+)= A[tmem] * B[smem desc], kind::f8f6f4 (e4m3 x e4m3), one CTA.
-__device__ __forceinline__ void mma_ts_f8(uint32_t d, uint32_t a, uint64_t bdesc, uint32_t idesc, uint32_t accum) {
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d),
-        "r"(a), "l"(bdesc), "r"(idesc), "r"(accum)
-        : "memory");
-}
-__device__ __forceinline__ void mma_commit(uint32_t bar) {
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
-                 : "memory");
-}
-
-#define EMTK_R16(r, o)                                                                                       \
-    "=r"(r[o + 0]), "=r"(r[o + 1]), "=r"(r[o + 2]), "=r"(r[o + 3]), "=r"(r[o + 4]), "=r"(r[o + 5]),         \
-        "=r"(r[o + 6]), "=r"(r[o + 7]), "=r"(r[o + 8]), "=r"(r[o + 9]), "=r"(r[o + 10]), "=r"(r[o + 11]), \
-        "=r"(r[o + 12]), "=r"(r[o + 13]), "=r"(r[o + 14]), "=r"(r[o + 15])
-
-template <int O, int N>
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[N]) {
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-        : EMTK_R16(r, O)
-        : "r"(taddr));
-}
-__device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
-__device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
-
-template <int O, int N>
-__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[N]) {
-    asm volatile(
-        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
-            taddr),
-        "r"(r[O + 0]), "r"(r[O + 1]), "r"(r[O + 2]), "r"(r[O + 3]), "r"(r[O + 4]), "r"(r[O + 5]), "r"(r[O + 6]),
-        "r"(r[O + 7]), "r"(r[O + 8]), "r"(r[O + 9]), "r"(r[O + 10]), "r"(r[O + 11]), "r"(r[O + 12]), "r"(r[O + 13]),
-        "r"(r[O + 14]), "r"(r[O + 15])
-        : "memory");
-}
-template <int O, int N>
-__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&r)[N]) {
-    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr), "r"(r[O + 0]),
-                 "r"(r[O + 1]), "r"(r[O + 2]), "r"(r[O + 3]), "r"(r[O + 4]), "r"(r[O + 5]), "r"(r[O + 6]),
-                 "r"(r[O + 7])
-                 : "memory");
-}
-// Makes later uses of r depend on the preceding tcgen05.wait::ld.
-template <int N>
-__device__ __forceinline__ void reg_fence(uint32_t (&r)[N]) {
-#pragma unroll
-    for (int i = 0; i < N; ++i) asm volatile("" : "+r"(r[i]));
-}
-
-template <bool FP16>
-__device__ __forceinline__ uint32_t relu_pack(uint32_t lo, uint32_t hi) {
-    uint32_t d;
-    if (FP16)
-        asm("cvt.rn.relu.f16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(__uint_as_float(hi)), "f"(__uint_as_float(lo)));
-    else
-        asm("cvt.rn.relu.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(__uint_as_float(hi)), "f"(__uint_as_float(lo)));
-    return d;
-}
-
-// ReLU of four fp32 values as four e4m3 bytes of one word, element 0 in the
-// lowest byte; satfinite clamps to 448.
-__device__ __forceinline__ uint32_t relu_e4m3x4(uint32_t v0, uint32_t v1, uint32_t v2, uint32_t v3) {
-    uint32_t r;
-    asm("{\n\t.reg .b16 lo, hi;\n\t"
-        "cvt.rn.satfinite.relu.e4m3x2.f32 lo, %2, %1;\n\t"
-        "cvt.rn.satfinite.relu.e4m3x2.f32 hi, %4, %3;\n\t"
-        "mov.b32 %0, {lo, hi};\n\t}"
-        : "=r"(r)
-        : "f"(__uint_as_float(v0)), "f"(__uint_as_float(v1)), "f"(__uint_as_float(v2)), "f"(__uint_as_float(v3)));
-    return r;
-}
-
-// Instruction descriptor, kind::f16: fp32 accumulate, both operands K-major.
-// With fp16 = true the format codes (0) are also those of e4m3 x e4m3 for
-// kind::f8f6f4.
-__host__ __device__ constexpr uint32_t make_idesc(int M, int N, bool fp16) {
-    return (1u << 4) | ((fp16 ? 0u : 1u) << 7) | ((fp16 ? 0u : 1u) << 10) | ((uint32_t)(N >> 3) << 17) |
-           ((uint32_t)(M >> 4) << 24);
-}
-
-// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups
-// 1024 bytes apart (SBO), sm_100 descriptor version.
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
-    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
-           ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
-}
-// The same for a 64-byte swizzle: 64-byte rows, 8-row groups 512 bytes apart.
-__device__ __forceinline__ uint64_t sw64_desc(uint32_t saddr) {
-    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) | ((uint64_t)(512 >> 4) << 32) |
-           ((uint64_t)1 << 46) | ((uint64_t)4 << 61);
-}
 
 // One 48-wide row of a hit's window, 16-bit pixels packed two per word:
 // element e0 of src and the 47 after it.  Seven aligned 16-byte loads cover
@@ -871,7 +674,7 @@ cudaError_t prepare_tc_weights(DeviceWeights &w, const emtk_weights &hw, TcMode 
     e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &qr);
     if (e != cudaSuccess || fn == nullptr || qr != cudaDriverEntryPointSuccess) return cudaErrorNotSupported;
     auto encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
-    CUtensorMap *map = new CUtensorMap;
+    CUtensorMap *map = new CUtensorMap[1];
     cuuint64_t dims[3] = {(cuuint64_t)kW1Box, (cuuint64_t)kN1, (cuuint64_t)kKBlocks};
     const cuuint64_t esz = f8 ? 1 : 2;  // bytes per weight
     cuuint64_t strides[2] = {(cuuint64_t)kW1Box * esz, (cuuint64_t)kW1Box * kN1 * esz};
@@ -883,7 +686,7 @@ cudaError_t prepare_tc_weights(DeviceWeights &w, const emtk_weights &hw, TcMode 
                         f8 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) {
-        delete map;
+        delete[] map;
         return cudaErrorInvalidValue;
     }
     w.w1_tmap = map;
@@ -912,6 +715,8 @@ cudaError_t launch_cnn_tc(const DeviceWeights &w, const void *src, const HitDesc
     const long long units = (long long)((n + 127) / 128) * kW1Steps;
     const uint16_t *src16 = static_cast<const uint16_t *>(src);
     dim3 grid(G);
+    if (mode == kTcSplit)
+        return launch_cnn_split(w, src, desc, n, G, partials, n_pad, status, timeout_ns, debug_stall, s);
     switch (mode) {
     case kTcFp16:
         cnn_tc_kernel<kTcFp16><<<grid, kThreadsTC, kSmemBytesTC, s>>>(

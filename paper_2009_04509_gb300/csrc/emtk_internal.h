@@ -124,18 +124,29 @@ struct DeviceWeights {
     float *mic_w = nullptr;      // [32]
     float *mic_b = nullptr;
     void *w1_tiles = nullptr;      // dense-1 weights, tiled for TMA: [1452][128][64] of 16 bit or e4m3
+                                   // (EMTK_TF32: fp16 heads, then fp16 tails, each so tiled)
     uint16_t *convB = nullptr;     // 16-bit conv B operand: [48][32] (taps 0-24, bias hi, bias lo, zeros)
-    void *w1_tmap = nullptr;       // host copy of the TMA descriptor (CUtensorMap, 128 B)
+    void *w1_tmap = nullptr;       // host copies of the TMA descriptors (CUtensorMap[1], or [2]: heads, tails)
     float fc1_scale = 1.0f;        // dense-1 sums are scaled by this before the bias (EMTK_FP8: 1/(s_a s_w))
-    float fc1_w_scale = 1.0f;      // EMTK_FP8: s_w, the power of two the weights were scaled by
+    float fc1_w_scale = 1.0f;      // EMTK_FP8 / EMTK_TF32: s_w, the power of two the weights were scaled by
+    float act_mul = 1.0f;          // EMTK_TF32: s_a / (s_p s_c), applied to the ReLU'd conv sums
     // host copy of the conv weights [25][48] and bias [48]: the fp32 kernel takes
     // them as a launch parameter (constant bank)
     float conv_w_host[kK * kK * kF] = {};
     float conv_b_host[kF] = {};
 };
 
-// Operand formats of the tensor-core kernel.
-enum TcMode { kTcBf16 = 0, kTcFp16 = 1, kTcFp8 = 2 };
+// Operand formats of the tensor-core kernels: 16-bit (cnn_tc.cu, also with
+// an e4m3 dense-1), and fp32 operands split into fp16 heads and tails
+// (cnn_split.cu, EMTK_TF32).
+enum TcMode { kTcBf16 = 0, kTcFp16 = 1, kTcFp8 = 2, kTcSplit = 3 };
+
+// Internal patch / interval-image format of EMTK_TF32: one 32-bit word per
+// pixel, the fp16 head of (value x kSplitPatchScale) in the low half and the
+// fp16 tail (the rest, rounded to fp16) in the high half.  Not a format of
+// the public emtk_patch_format.
+constexpr emtk_patch_format kPatchSplit16 = static_cast<emtk_patch_format>(3);
+constexpr float kSplitPatchScale = 0.0625f;  // s_p: 2^-4
 
 }  // namespace emtk
 
@@ -252,8 +263,13 @@ cudaError_t init_fp32_kernel_attrs();
 cudaError_t init_head_kernel_attrs();
 cudaError_t init_tc_kernel_attrs();
 
-// Host helpers for the tensor-core weights (cnn_tc.cu).
+// Host helpers for the tensor-core weights (cnn_tc.cu, cnn_split.cu).
 cudaError_t prepare_tc_weights(DeviceWeights &w, const emtk_weights &hw, TcMode mode);
+cudaError_t prepare_split_weights(DeviceWeights &w, const emtk_weights &hw);
+cudaError_t init_split_kernel_attrs();
+cudaError_t launch_cnn_split(const DeviceWeights &w, const void *src, const HitDesc *desc, int32_t n, int G,
+                             float *partials, int n_pad, int *status, int64_t timeout_ns, int debug_stall,
+                             cudaStream_t s);
 // EMTK_FP8 weight scale: the largest power of two s_w with max|W1| s_w <= 448.
 double fp8_weight_scale(const float *fc1_w, size_t n);
 int choose_splits_fp32(int n, int sm_count, int max_splits);

@@ -28,9 +28,26 @@ __device__ __forceinline__ float interval_sum(float a0, float a1, float a2, floa
     return __fdiv_rn(s, 6.0f);
 }
 
+// One pixel of the EMTK_TF32 image: the fp16 head of v * s_p in the low half,
+// the fp16 tail (v * s_p - head, rounded) in the high half.  s_p is a power
+// of two, so the product is exact.
+__device__ __forceinline__ uint32_t split_word(float v) {
+    const float x = __fmul_rn(v, kSplitPatchScale);
+    const __half h = __float2half_rn(x);
+    const __half t = __float2half_rn(__fsub_rn(x, __half2float(h)));
+    return (uint32_t)__half_as_ushort(h) | ((uint32_t)__half_as_ushort(t) << 16);
+}
+
 template <int FMT>
 __device__ __forceinline__ void store2(void *base, int64_t idx, float v0, float v1, bool two) {
-    if (FMT == EMTK_PATCH_F32) {
+    if (FMT == kPatchSplit16) {
+        uint32_t *p = static_cast<uint32_t *>(base) + idx;
+        if (two) {
+            *reinterpret_cast<uint2 *>(p) = make_uint2(split_word(v0), split_word(v1));
+        } else {
+            p[0] = split_word(v0);
+        }
+    } else if (FMT == EMTK_PATCH_F32) {
         float *p = static_cast<float *>(base) + idx;
         if (two) {
             *reinterpret_cast<float2 *>(p) = make_float2(v0, v1);
@@ -171,7 +188,9 @@ template <int FMT>
 __global__ void convert_kernel(const float *src, void *dst, int64_t n) {
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
         const float v = src[i];
-        if (FMT == EMTK_PATCH_BF16)
+        if (FMT == kPatchSplit16)
+            static_cast<uint32_t *>(dst)[i] = split_word(v);
+        else if (FMT == EMTK_PATCH_BF16)
             static_cast<__nv_bfloat16 *>(dst)[i] = __float2bfloat16_rn(v);
         else
             static_cast<__half *>(dst)[i] = __float2half_rn(v);
@@ -244,7 +263,10 @@ cudaError_t launch_interval_images(const ReqTable &t, void *dimg, emtk_patch_for
         int64_t bx = (want + 255) / 256;
         if (bx > 4096) bx = 4096;
         dim3 grid((unsigned)bx, (unsigned)t.n + 1);
-        if (fmt == EMTK_PATCH_F32)
+        if (fmt == kPatchSplit16)
+            interval_desc_kernel<kPatchSplit16><<<grid, 256, 0, s>>>(t, dimg, job->g0, job->count, job->desc,
+                                                                     job->dest, job->out_stride);
+        else if (fmt == EMTK_PATCH_F32)
             interval_desc_kernel<EMTK_PATCH_F32><<<grid, 256, 0, s>>>(t, dimg, job->g0, job->count, job->desc,
                                                                       job->dest, job->out_stride);
         else if (fmt == EMTK_PATCH_BF16)
@@ -259,7 +281,9 @@ cudaError_t launch_interval_images(const ReqTable &t, void *dimg, emtk_patch_for
     int64_t bx = (most + 255) / 256;
     if (bx > 4096) bx = 4096;
     dim3 grid((unsigned)bx, (unsigned)t.n);
-    if (fmt == EMTK_PATCH_F32)
+    if (fmt == kPatchSplit16)
+        interval_image_kernel<kPatchSplit16><<<grid, 256, 0, s>>>(t, dimg);
+    else if (fmt == EMTK_PATCH_F32)
         interval_image_kernel<EMTK_PATCH_F32><<<grid, 256, 0, s>>>(t, dimg);
     else if (fmt == EMTK_PATCH_BF16)
         interval_image_kernel<EMTK_PATCH_BF16><<<grid, 256, 0, s>>>(t, dimg);
@@ -284,7 +308,9 @@ cudaError_t launch_convert_patches(const float *src, void *dst, emtk_patch_forma
     if (n <= 0) return cudaSuccess;
     int64_t blocks = (n + 255) / 256;
     if (blocks > 8192) blocks = 8192;
-    if (fmt == EMTK_PATCH_BF16)
+    if (fmt == kPatchSplit16)
+        convert_kernel<kPatchSplit16><<<(unsigned)blocks, 256, 0, s>>>(src, dst, n);
+    else if (fmt == EMTK_PATCH_BF16)
         convert_kernel<EMTK_PATCH_BF16><<<(unsigned)blocks, 256, 0, s>>>(src, dst, n);
     else
         convert_kernel<EMTK_PATCH_F16><<<(unsigned)blocks, 256, 0, s>>>(src, dst, n);

@@ -30,7 +30,7 @@ def main() -> int:
     ap = argparse.ArgumentParser()
     ap.add_argument("--mode", default="event", choices=["event", "patches", "hitfind"])
     ap.add_argument("--hits", type=int, default=30000, help="patches mode: number of patches")
-    ap.add_argument("--precision", default="bf16", choices=["bf16", "fp16", "fp8", "fp32"])
+    ap.add_argument("--precision", default="bf16", choices=["bf16", "fp16", "fp8", "fp32", "tf32"])
     ap.add_argument("--runs", type=int, default=2)
     args = ap.parse_args()
 

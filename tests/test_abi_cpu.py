@@ -113,8 +113,8 @@ def test_argument_errors_without_device(lib):
     o.max_hits = 0
     assert lib.emtk_create(ctypes.byref(ws), ctypes.byref(o), 0, ctypes.byref(out)) == emtk.EMTK_ERR_ARG
     o = emtk.emtk_default_options()
-    o.precision = emtk.EMTK_TF32
-    assert lib.emtk_create(ctypes.byref(ws), ctypes.byref(o), 0, ctypes.byref(out)) == emtk.EMTK_ERR_UNSUPPORTED
+    o.debug_stall = 2
+    assert lib.emtk_create(ctypes.byref(ws), ctypes.byref(o), 0, ctypes.byref(out)) == emtk.EMTK_ERR_ARG
     assert lib.emtk_create(ctypes.byref(ws), None, -1, ctypes.byref(out)) == emtk.EMTK_ERR_ARG
 
 
@@ -125,6 +125,26 @@ def test_create_without_gpu_reports_cuda_error(lib):
     with pytest.raises(emtk.EmtkError) as e:
         emtk.emtk_create(synth.he_normal_weights(0), precision="bf16")
     assert e.value.status == emtk.EMTK_ERR_CUDA
+
+
+def test_every_precision_is_accepted_then_needs_a_device(lib):
+    """All five precisions are valid arguments (EMTK_TF32 included); without a
+    GPU, creation fails at the device, not at the argument check."""
+    torch = pytest.importorskip("torch")
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    for prec in ("fp32", "tf32", "bf16", "fp16", "fp8"):
+        with pytest.raises(emtk.EmtkError) as e:
+            emtk.emtk_create(synth.he_normal_weights(0), precision=prec)
+        assert e.value.status == emtk.EMTK_ERR_CUDA, prec
+
+
+def test_fault_injection_hooks_without_device(lib):
+    """The test hooks are host-only: they work without a device."""
+    emtk.emtk_debug_fail_alloc(3)
+    emtk.emtk_debug_fail_alloc(-1)
+    assert emtk.emtk_debug_alloc_counts() == (0, 0)
+    assert lib.emtk_debug_batcher_stall(None, 1) == emtk.EMTK_ERR_ARG
 
 
 def test_missing_library_fails_loudly(tmp_path):

@@ -9,8 +9,9 @@ conv weights, post-ReLU activations and dense-1 weights to bf16 / fp16, or
 the dense-1 operands to e4m3 with the same power-of-two scales).  Bars:
 
 * every path: finite scores, softmax rows summing to 1, scores in [0, 1];
-* fp32: max |score - fp64| <= 1e-3 on every hit, and every logit within
-  TOL_LOGIT_FP32 (1 + |z|) of the fp64 logit;
+* fp32 and tf32 (the fp32-accuracy paths): max |score - fp64| <= 1e-3 on
+  every hit, and every logit within TOL_LOGIT_FP32 (1 + |z|) of the fp64
+  logit;
 * bf16 / fp16: argmax agreement with fp64 >= 99.5% over all 60,000 hits;
   max |score - emulation| <= 2e-2 on every hit; every logit within
   TOL_LOGIT_16 (1 + |z|) of the emulation's;
@@ -117,8 +118,11 @@ def logit_err(z, ref):
     return float((np.abs(z - ref) / (1.0 + np.abs(ref))).max())
 
 
-def test_full_event_fp32_every_hit(emtk, event):
-    s, z = run_event(emtk, event, "fp32")
+@pytest.mark.parametrize("prec", ["fp32", "tf32"])
+def test_full_event_fp32_every_hit(emtk, event, prec):
+    """The fp32 bar for both fp32-accuracy paths: CUDA-core fp32 and the
+    tensor-core split-fp16 path (EMTK_TF32)."""
+    s, z = run_event(emtk, event, prec)
     lo, ref = event["fp64"]
     d = np.abs(s - ref)
     assert d.max() <= TOL_FP32, f"max |score - fp64| = {d.max():.3g} at hit {np.unravel_index(d.argmax(), d.shape)}"

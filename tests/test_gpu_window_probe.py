@@ -19,6 +19,11 @@ exact, decodable function of known window pixels:
   sum_k 2^(4k-8) p_k exactly (fewer than 24 significant bits);
 * dense-2 and the heads pass neuron L through to logit L.
 
+In tf32 (split fp16 heads and tails) every value above is an fp16 head with
+a zero tail, after the power-of-two scales, so the sums stay exact; that
+path reads its windows with code of its own (32-bit pixels), probed here over
+every pixel as bf16's is.
+
 The logits must then equal, bit for bit, the same sums of the oracle's patch
 pixels; the oracle's own fp64 network on the same weights must agree too
 (a check of the test's decoding).  Across the contexts every pixel of the
@@ -121,7 +126,7 @@ def expected_logits(patches, where, n):
     return z
 
 
-@pytest.mark.parametrize("prec", ["bf16", "fp16", "fp8"])
+@pytest.mark.parametrize("prec", ["bf16", "fp16", "fp8", "tf32"])
 def test_window_read_bit_exact(emtk, prec):
     adc_np, _ = probe_plane()
     hits_np = probe_hits()
@@ -134,8 +139,8 @@ def test_window_read_bit_exact(emtk, prec):
     patches = torch.from_numpy(want_p).cuda()
     per_logit = 3 if prec == "fp8" else 6
     groups = probe_pixels(per_logit)
-    if prec != "bf16":
-        groups = groups[::7]               # the window read is the same code in every mode
+    if prec in ("fp16", "fp8"):
+        groups = groups[::7]               # the window read of bf16, fp16 and fp8 is one code
     for gi, pixels in enumerate(groups):
         w, where = probe_weights(pixels, per_logit)
         ctx = emtk.emtk_create(w, precision=prec, debug_logits=True, max_hits=256)
