@@ -26,10 +26,12 @@
 // Work units, stream-K split and warp roles are those of cnn_tc.cu.  The
 // differences:
 //   builder warps   an interval-image pixel is a 32-bit word (fp16 head in
-//                   the low half, tail in the high half).  A thread reads its
-//                   hit's 5 x 8 window words of each quad (a whole window row
-//                   of words does not fit the registers) and writes two
-//                   im2col tiles, heads and tails;
+//                   the low half, tail in the high half).  A whole window row
+//                   of words does not fit the registers, so a thread slides
+//                   along each output row instead: it keeps the 16-byte chunks
+//                   the next quad shares with this one and loads one new chunk
+//                   per window row, a quad ahead; it writes two im2col tiles,
+//                   heads and tails;
 //   conv issuer     6 MMAs per pair (heads x head weights, heads x tail
 //                   weights, tails x head weights; K = 32 each, as two K16);
 //   epilogue        each position's 48 fp32 conv sums become 48 fp16 heads
@@ -118,31 +120,8 @@ __device__ __forceinline__ void split2(float v0, float v1, uint32_t &head, uint3
     asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(tail) : "f"(__fsub_rn(v1, h1)), "f"(__fsub_rn(v0, h0)));
 }
 
-// Words e .. e+7 of the image (each pixel one word).  Aligned 16-byte loads,
-// then a shift by e % 4 words made of selects; src must have 16 bytes of
-// readable memory past word e + 7.
-__device__ __forceinline__ void load_words8(const uint32_t *__restrict__ src, int64_t e, uint32_t (&out)[8]) {
-    const int m = (int)(e & 3);
-    const uint4 *p = reinterpret_cast<const uint4 *>(src + (e - m));
-    uint32_t w[12];
-    const uint4 a = __ldg(p), b = __ldg(p + 1);
-    w[0] = a.x, w[1] = a.y, w[2] = a.z, w[3] = a.w, w[4] = b.x, w[5] = b.y, w[6] = b.z, w[7] = b.w;
-    if (m == 0) {
-#pragma unroll
-        for (int j = 0; j < 8; ++j) out[j] = w[j];
-        return;
-    }
-    const uint4 c = __ldg(p + 2);
-    w[8] = c.x, w[9] = c.y, w[10] = c.z, w[11] = c.w;
-    uint32_t s2[10];
-#pragma unroll
-    for (int j = 0; j < 10; ++j) s2[j] = (m & 2) ? w[j + 2] : w[j];
-#pragma unroll
-    for (int j = 0; j < 8; ++j) out[j] = (m & 1) ? s2[j + 1] : s2[j];
-}
-
-// The same words of window row r, columns x0 .. x0+7, for a hit whose window
-// leaves the haloed image: every pixel checked against the plane, zero outside.
+// Words x0 .. x0+7 of window row r for a hit whose window leaves the haloed
+// image: every pixel checked against the plane, zero outside.
 __device__ __forceinline__ void load_words8_checked(const uint32_t *__restrict__ src, const HitDesc &hd, int r,
                                                    int x0, uint32_t (&out)[8]) {
     const int w = hd.wc - kHalf + r;
@@ -383,18 +362,70 @@ __global__ void __launch_bounds__(kThreadsSp, 1)
             } else {
                 hd.inside = 1;
             }
+            // The window words of a quad at x0 lie in 16-byte chunks eb, eb+4 and, for
+            // a window not aligned to 4 words (m > 0), eb+8 of each of its 5 rows
+            // (eb = first word of the row + x0 - m).  Consecutive quads of an
+            // output row share all but the last chunk, so `raw` carries them and
+            // the new chunk of the next quad is loaded into `nxt` while this one
+            // is built.
+            const int m = (int)(hd.origin & 3);
+            const bool fast = valid && hd.inside;
+            uint32_t raw[kK][12], nxt[kK][4];
             for (int quad = j0; ok && quad < j1; ++quad) {
                 const int y = quad / (kQ / 4), x0 = 4 * (quad % (kQ / 4));
                 uint32_t W[kK][8];
+                if (fast) {
+                    const int64_t eb0 = hd.origin + (int64_t)y * hd.pitch + x0 - m;
+                    if (quad == j0 || x0 == 0) {  // a new output row: load the chunks
 #pragma unroll
-                for (int i = 0; i < kK; ++i) {
-                    if (!valid) {
+                        for (int i = 0; i < kK; ++i) {
+                            const uint4 *pc = reinterpret_cast<const uint4 *>(src + eb0 + (int64_t)i * hd.pitch);
+                            const uint4 c0 = __ldg(pc), c1 = __ldg(pc + 1);
+                            raw[i][0] = c0.x, raw[i][1] = c0.y, raw[i][2] = c0.z, raw[i][3] = c0.w;
+                            raw[i][4] = c1.x, raw[i][5] = c1.y, raw[i][6] = c1.z, raw[i][7] = c1.w;
+                            if (m != 0) {
+                                const uint4 c2 = __ldg(pc + 2);
+                                raw[i][8] = c2.x, raw[i][9] = c2.y, raw[i][10] = c2.z, raw[i][11] = c2.w;
+                            }
+                        }
+                    } else {  // one chunk further: the prefetched one comes last
 #pragma unroll
-                        for (int j = 0; j < 8; ++j) W[i][j] = 0u;
-                    } else if (hd.inside) {
-                        load_words8(src, hd.origin + (int64_t)(y + i) * hd.pitch + x0, W[i]);
-                    } else {
-                        load_words8_checked(src, hd, y + i, x0, W[i]);
+                        for (int i = 0; i < kK; ++i) {
+#pragma unroll
+                            for (int j = 0; j < 4; ++j) {
+                                raw[i][j] = raw[i][j + 4];
+                                raw[i][j + 4] = m != 0 ? raw[i][j + 8] : nxt[i][j];
+                                raw[i][j + 8] = nxt[i][j];
+                            }
+                        }
+                    }
+                    // the next quad of this output row: its new chunk, ahead of time
+                    if (quad + 1 < j1 && x0 + 4 < kQ) {
+                        const int64_t nc = eb0 + (m != 0 ? 12 : 8);
+#pragma unroll
+                        for (int i = 0; i < kK; ++i) {
+                            const uint4 v = __ldg(reinterpret_cast<const uint4 *>(src + nc + (int64_t)i * hd.pitch));
+                            nxt[i][0] = v.x, nxt[i][1] = v.y, nxt[i][2] = v.z, nxt[i][3] = v.w;
+                        }
+                    }
+                    // words m .. m+7 of each row: a shift made of selects
+#pragma unroll
+                    for (int i = 0; i < kK; ++i) {
+                        uint32_t s2[10];
+#pragma unroll
+                        for (int j = 0; j < 10; ++j) s2[j] = (m & 2) ? raw[i][j + 2] : raw[i][j];
+#pragma unroll
+                        for (int j = 0; j < 8; ++j) W[i][j] = (m & 1) ? s2[j + 1] : s2[j];
+                    }
+                } else {
+#pragma unroll
+                    for (int i = 0; i < kK; ++i) {
+                        if (valid) {
+                            load_words8_checked(src, hd, y + i, x0, W[i]);
+                        } else {
+#pragma unroll
+                            for (int j = 0; j < 8; ++j) W[i][j] = 0u;
+                        }
                     }
                 }
                 const int k = (int)(k_base + quad);
