@@ -162,6 +162,8 @@ __global__ void __launch_bounds__(kThreadsSp, 1)
     const int tile0 = (int)(u0 / kQuads);
     const Guard guard{abort_flag, status, (int64_t)timeout_ns};
 
+    // the next kernel (the head) may be scheduled as SMs free up; it waits for this one
+    pdl_trigger();
     // ---- set-up: conv B heads and tails into 64-byte-swizzled smem, barriers, TMEM
     for (int idx = threadIdx.x; idx < 2 * kPairNSp * 4; idx += kThreadsSp) {
         const int h = idx / (kPairNSp * 4), rem = idx % (kPairNSp * 4);
@@ -342,6 +344,7 @@ __global__ void __launch_bounds__(kThreadsSp, 1)
         const int q4 = builder_of(warp);
         const int row = 32 * q4 + lane;
         constexpr uint32_t ones = 0x3C003C00u;  // two fp16 1.0
+        pdl_wait();  // the images and window descriptors come from the kernel before
         uint8_t *my_hi = gbase + kOffImSp + row * 128;
         bool ok = true;
         const int t_first = tile0;
@@ -660,10 +663,12 @@ cudaError_t launch_cnn_split(const DeviceWeights &w, const void *src, const HitD
     if (n <= 0) return cudaSuccess;
     const CUtensorMap *maps = static_cast<const CUtensorMap *>(w.w1_tmap);
     const long long units = (long long)((n + 127) / 128) * kQuads;
-    cnn_split_kernel<<<G, kThreadsSp, kSmemBytesSp, s>>>(maps[0], maps[1], static_cast<const uint32_t *>(src), desc,
-                                                         n, w.convB, w.act_mul, partials, n_pad, units, status,
-                                                         (long long)timeout_ns, debug_stall);
-    return cudaGetLastError();
+    const uint32_t *src32 = static_cast<const uint32_t *>(src);
+    const uint16_t *convB = w.convB;
+    const float act_mul = w.act_mul;
+    const long long tmo = (long long)timeout_ns;
+    return launch_pdl(cnn_split_kernel, dim3(G), dim3(kThreadsSp), kSmemBytesSp, s, maps[0], maps[1], src32, desc, n,
+                      convB, act_mul, partials, n_pad, units, status, tmo, debug_stall);
 }
 
 }  // namespace emtk

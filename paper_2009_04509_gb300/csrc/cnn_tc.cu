@@ -197,6 +197,8 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     constexpr int kStageTx = F8 ? kW1StageBytesF8 : kW1StageBytes;
     constexpr int kBoxTx = F8 ? kW1BoxBytesF8 : kW1BoxBytes;
 
+    // the next kernel (the head) may be scheduled as SMs free up; it waits for this one
+    pdl_trigger();
     // ---- set-up: pair conv B operand into swizzled smem, barriers, TMEM
     for (int idx = threadIdx.x; idx < kPairN * 8; idx += kThreadsTC) {
         const int row = idx >> 3, chunk = idx & 7;
@@ -391,6 +393,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         const int q4 = builder_index(warp);
         const int row = 32 * q4 + lane;
         const uint32_t one = FP16 ? 0x3C00u : 0x3F80u;
+        pdl_wait();  // the images and window descriptors come from the kernel before
         const uint32_t ones = one | (one << 16);
         uint8_t *my_row = gbase + kOffIm + row * 128;
         bool ok = true;
@@ -717,21 +720,12 @@ cudaError_t launch_cnn_tc(const DeviceWeights &w, const void *src, const HitDesc
     dim3 grid(G);
     if (mode == kTcSplit)
         return launch_cnn_split(w, src, desc, n, G, partials, n_pad, status, timeout_ns, debug_stall, s);
-    switch (mode) {
-    case kTcFp16:
-        cnn_tc_kernel<kTcFp16><<<grid, kThreadsTC, kSmemBytesTC, s>>>(
-            map, src16, desc, n, w.convB, partials, n_pad, units, status, (long long)timeout_ns, debug_stall);
-        break;
-    case kTcFp8:
-        cnn_tc_kernel<kTcFp8><<<grid, kThreadsTC, kSmemBytesTC, s>>>(
-            map, src16, desc, n, w.convB, partials, n_pad, units, status, (long long)timeout_ns, debug_stall);
-        break;
-    default:
-        cnn_tc_kernel<kTcBf16><<<grid, kThreadsTC, kSmemBytesTC, s>>>(
-            map, src16, desc, n, w.convB, partials, n_pad, units, status, (long long)timeout_ns, debug_stall);
-        break;
-    }
-    return cudaGetLastError();
+    auto *kernel = mode == kTcFp16 ? cnn_tc_kernel<kTcFp16> : mode == kTcFp8 ? cnn_tc_kernel<kTcFp8>
+                                                                              : cnn_tc_kernel<kTcBf16>;
+    const uint16_t *convB = w.convB;
+    const long long tmo = (long long)timeout_ns;
+    return launch_pdl(kernel, grid, dim3(kThreadsTC), kSmemBytesTC, s, map, src16, desc, n, convB, partials, n_pad,
+                      units, status, tmo, debug_stall);
 }
 
 }  // namespace emtk

@@ -148,6 +148,33 @@ enum TcMode { kTcBf16 = 0, kTcFp16 = 1, kTcFp8 = 2, kTcSplit = 3 };
 constexpr emtk_patch_format kPatchSplit16 = static_cast<emtk_patch_format>(3);
 constexpr float kSplitPatchScale = 0.0625f;  // s_p: 2^-4
 
+// Programmatic dependent launch.  A kernel launched with launch_pdl may
+// start before the kernel before it on the stream has completed (once every
+// CTA of that one has started and executed pdl_trigger, or finished), so its
+// set-up overlaps that kernel's tail; before it reads anything that kernel
+// (or an earlier one) wrote, it executes pdl_wait, which returns once the
+// previous kernel has completed and its writes are visible.
+#ifdef __CUDACC__
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+#endif
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                       Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args &&>(args)...);
+}
+
 }  // namespace emtk
 
 struct emtk_pending_event {

@@ -111,6 +111,7 @@ __device__ __forceinline__ void interval_request(const ReqDesc &r, void *img) {
 // grid.y = request.
 template <int FMT>
 __global__ void __launch_bounds__(256) interval_image_kernel(const __grid_constant__ ReqTable t, void *img) {
+    pdl_trigger();  // the network kernel may set up while this one finishes; it waits for it
     interval_request<FMT>(t.r[blockIdx.y], img);
 }
 
@@ -222,6 +223,7 @@ __device__ __forceinline__ void hit_desc_one(const ReqTable &t, int64_t g0, int6
 
 __global__ void hit_desc_kernel(const __grid_constant__ ReqTable t, int64_t g0, int32_t count, HitDesc *desc,
                                 float **dest, int out_stride) {
+    pdl_trigger();
     const int64_t local = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (local < count) hit_desc_one(t, g0, local, desc, dest, out_stride);
 }
@@ -233,6 +235,7 @@ template <int FMT>
 __global__ void __launch_bounds__(256) interval_desc_kernel(const __grid_constant__ ReqTable t, void *img, int64_t g0,
                                                             int32_t count, HitDesc *desc, float **dest,
                                                             int out_stride) {
+    pdl_trigger();
     if ((int)blockIdx.y < t.n) {
         interval_request<FMT>(t.r[blockIdx.y], img);
         return;
@@ -243,6 +246,7 @@ __global__ void __launch_bounds__(256) interval_desc_kernel(const __grid_constan
 }
 
 __global__ void fill_dest_kernel(float *scores, int stride, float **dest, int32_t n) {
+    pdl_trigger();
     const int i = blockIdx.x * blockDim.x + threadIdx.x;
     if (i < n) dest[i] = scores + (int64_t)i * stride;
 }

@@ -4,12 +4,16 @@
 // head (track, em, none) and the Michel sigmoid head.  The rows of a hit are
 // the K-splits of the fp32 path, or the stream-K CTAs that shared its tile.
 // Three kernels, chosen by launch_head, with the same sums in the same order
-// (so the same bits):
+// (so the same bits), except where noted:
 //   head_kernel       small launches with few rows: a thread per hit streams
 //                     its dense-1 outputs four at a time into the 32 dense-2
 //                     sums (weights broadcast from shared memory);
 //   head_rows_kernel  many rows per hit (small launches spread each tile
-//                     over many CTAs): a warp per hit sums the rows, 16 deep;
+//                     over many CTAs): a warp per hit sums the rows, 16 deep
+//                     (from 32 rows on, four warps per hit each sum a
+//                     quarter of the rows and the quarters are added in
+//                     order: the same bits run to run, a different rounding
+//                     order than the other two kernels);
 //   head_tile_kernel  large launches: one CTA per 128-hit tile (coalesced
 //                     row sums, a register-tiled dense-2).
 #include "emtk_internal.h"
@@ -33,6 +37,7 @@ __device__ __forceinline__ void stage_w2(float *w2, const float *__restrict__ fc
     for (int k = 0; k < kN4 / kThreads; ++k) reinterpret_cast<float4 *>(w2)[threadIdx.x + k * kThreads] = v[k];
 }
 constexpr int kManyRows = 4;  // above this many partial rows per hit, reduce them with a warp per hit
+constexpr int kSplitRows = 32;  // from this many, with four warps per hit
 
 __global__ void __launch_bounds__(kThreadsHead) head_kernel(const float *__restrict__ partials, int splits, int G,
                                                            int n_pad, int32_t n, float s1,
@@ -55,6 +60,7 @@ __global__ void __launch_bounds__(kThreadsHead) head_kernel(const float *__restr
         b2[i] = fc2_b[i];
     }
     for (int i = threadIdx.x; i < kN1; i += blockDim.x) b1[i] = fc1_b[i];
+    pdl_wait();  // the partial sums and output rows come from the kernels before
     __syncthreads();
 
     const int64_t h = (int64_t)blockIdx.x * kThreadsHead + threadIdx.x;
@@ -135,7 +141,11 @@ constexpr int kThreadsRows = 256;
 constexpr int kSmallLaunch = 2048;
 constexpr int kH1Stride = kN1 + 1;  // shared h1 rows padded: thread t reads row t conflict-free
 
-template <int kHitsRows>
+// kSplit warps share a hit: warp k of the hit sums its rows [k R / kSplit,
+// (k+1) R / kSplit) in order, and the kSplit partial sums are then added in
+// k order (kSplit = 1: all rows in order, as head_kernel does).  More warps
+// per hit put more of the GPU on a small launch's many rows.
+template <int kHitsRows, int kSplit = 1>
 __global__ void __launch_bounds__(kThreadsRows) head_rows_kernel(const float *__restrict__ partials, int splits,
                                                                 int G, int n_pad, int32_t n, float s1,
                                                                 const float *__restrict__ fc1_b,
@@ -146,7 +156,9 @@ __global__ void __launch_bounds__(kThreadsRows) head_rows_kernel(const float *__
                                                                 const float *__restrict__ mic_w,
                                                                 const float *__restrict__ mic_b, float *const *dest,
                                                                 int debug_logits) {
+    static_assert(kHitsRows * kSplit <= kThreadsRows / 32 || kSplit == 1, "a warp per (hit, row share)");
     __shared__ float h1s[kHitsRows * kH1Stride];
+    __shared__ __align__(16) float4 part[kSplit > 1 ? kHitsRows * kSplit * 32 : 1];
     __shared__ float h2s[kHitsRows * (kN2 + 1)];
     __shared__ __align__(16) float w2[kN1][kN2];
     __shared__ __align__(16) float wc[kN2][kNC + 1];
@@ -158,25 +170,31 @@ __global__ void __launch_bounds__(kThreadsRows) head_rows_kernel(const float *__
         b2[i] = fc2_b[i];
     }
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    pdl_wait();  // the partial sums and output rows come from the kernels before
     const int64_t h0 = (int64_t)blockIdx.x * kHitsRows;
     const int64_t row_stride = (int64_t)n_pad * kN1 / 4;  // float4s between partial rows
     const float4 bb = reinterpret_cast<const float4 *>(fc1_b)[lane];
-    for (int j = warp; j < kHitsRows; j += kThreadsRows / 32) {
+    for (int jw = warp; jw < kHitsRows * kSplit; jw += kThreadsRows / 32) {
+        const int j = jw / kSplit, share = jw % kSplit;
         const int64_t h = h0 + j;
-        if (h >= n) break;
+        if (h >= n) {
+            if (kSplit > 1) continue;
+            break;
+        }
         int rows = splits;
         if (G > 0) {
             const int64_t units = (int64_t)((n + 127) / 128) * kQuads;
             const int64_t tile = h >> 7;
             rows = cta_of_unit(tile * kQuads + kQuads - 1, units, G) - cta_of_unit(tile * kQuads, units, G) + 1;
         }
+        const int r_end = (int)((int64_t)rows * (share + 1) / kSplit);
         const float4 *p = reinterpret_cast<const float4 *>(partials + h * kN1) + lane;
         float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
-        // rows in order (the same sum as head_kernel), loaded 16 at a time so that a
-        // hit with many rows waits for a few round trips, not one per row
+        // this warp's rows in order, loaded 16 at a time so that a hit with many
+        // rows waits for a few round trips, not one per row
         constexpr int kDepth = 16;
-        int r = 0;
-        for (; r + kDepth <= rows; r += kDepth) {
+        int r = (int)((int64_t)rows * share / kSplit);
+        for (; r + kDepth <= r_end; r += kDepth) {
             float4 v[kDepth];
 #pragma unroll
             for (int k = 0; k < kDepth; ++k) v[k] = p[(r + k) * row_stride];
@@ -188,18 +206,41 @@ __global__ void __launch_bounds__(kThreadsRows) head_rows_kernel(const float *__
                 a.w += v[k].w;
             }
         }
-        for (; r < rows; ++r) {
+        for (; r < r_end; ++r) {
             const float4 v = p[r * row_stride];
             a.x += v.x;
             a.y += v.y;
             a.z += v.z;
             a.w += v.w;
         }
+        if (kSplit > 1) {
+            part[jw * 32 + lane] = a;
+            continue;
+        }
         float *o = h1s + j * kH1Stride + 4 * lane;
         o[0] = fmaxf(fmaf(a.x, s1, bb.x), 0.f);
         o[1] = fmaxf(fmaf(a.y, s1, bb.y), 0.f);
         o[2] = fmaxf(fmaf(a.z, s1, bb.z), 0.f);
         o[3] = fmaxf(fmaf(a.w, s1, bb.w), 0.f);
+    }
+    if (kSplit > 1) {  // the shares of each hit, added in share order
+        __syncthreads();
+        for (int jw = warp; jw < kHitsRows; jw += kThreadsRows / 32) {
+            float4 a = part[(jw * kSplit) * 32 + lane];
+#pragma unroll
+            for (int k = 1; k < kSplit; ++k) {
+                const float4 v = part[(jw * kSplit + k) * 32 + lane];
+                a.x += v.x;
+                a.y += v.y;
+                a.z += v.z;
+                a.w += v.w;
+            }
+            float *o = h1s + jw * kH1Stride + 4 * lane;
+            o[0] = fmaxf(fmaf(a.x, s1, bb.x), 0.f);
+            o[1] = fmaxf(fmaf(a.y, s1, bb.y), 0.f);
+            o[2] = fmaxf(fmaf(a.z, s1, bb.z), 0.f);
+            o[3] = fmaxf(fmaf(a.w, s1, bb.w), 0.f);
+        }
     }
     __syncthreads();
     // dense-2 with every thread: output j of hit i is thread (32 i + j) mod 256's,
@@ -281,6 +322,7 @@ __global__ void __launch_bounds__(kThreadsTile) head_tile_kernel(const float *__
         wc[i][kNC] = mic_w[i];
         b2[i] = fc2_b[i];
     }
+    pdl_wait();  // the partial sums and output rows come from the kernels before
     const int64_t h0 = (int64_t)blockIdx.x * kTileHits;
     int rows = splits;
     if (G > 0) {
@@ -386,27 +428,25 @@ cudaError_t launch_head(const DeviceWeights &w, const float *partials, int split
     if (n <= 0) return cudaSuccess;
     // most partial rows a hit has: many when a small launch spreads each tile over many CTAs
     const int rows = G > 0 ? streamk_partial_rows(n, G) : splits;
+    // launched as dependents of the network kernel: the weights are staged while it finishes
+    const float s1 = w.fc1_scale;
+    const float *b1 = w.fc1_b, *w2 = w.fc2_w, *b2 = w.fc2_b, *wc = w.cls_w, *bc = w.cls_b, *wm = w.mic_w,
+                *bm = w.mic_b;
     if (rows > kManyRows) {
+        if (rows >= kSplitRows && n <= kSmallLaunch)  // a hit's rows over 4 warps, 2 hits per block
+            return launch_pdl(head_rows_kernel<2, 4>, dim3((n + 1) / 2), dim3(kThreadsRows), 0, s, partials, splits,
+                              G, n_pad, n, s1, b1, w2, b2, wc, bc, wm, bm, dest, debug_logits);
         if (n <= kSmallLaunch)
-            head_rows_kernel<8><<<(n + 7) / 8, kThreadsRows, 0, s>>>(
-                partials, splits, G, n_pad, n, w.fc1_scale, w.fc1_b, w.fc2_w, w.fc2_b, w.cls_w, w.cls_b, w.mic_w,
-                w.mic_b, dest, debug_logits);
-        else
-            head_rows_kernel<32><<<(n + 31) / 32, kThreadsRows, 0, s>>>(
-                partials, splits, G, n_pad, n, w.fc1_scale, w.fc1_b, w.fc2_w, w.fc2_b, w.cls_w, w.cls_b, w.mic_w,
-                w.mic_b, dest, debug_logits);
-        return cudaGetLastError();
+            return launch_pdl(head_rows_kernel<8>, dim3((n + 7) / 8), dim3(kThreadsRows), 0, s, partials, splits, G,
+                              n_pad, n, s1, b1, w2, b2, wc, bc, wm, bm, dest, debug_logits);
+        return launch_pdl(head_rows_kernel<32>, dim3((n + 31) / 32), dim3(kThreadsRows), 0, s, partials, splits, G,
+                          n_pad, n, s1, b1, w2, b2, wc, bc, wm, bm, dest, debug_logits);
     }
-    if (n > kSmallLaunch) {
-        head_tile_kernel<<<(n + kTileHits - 1) / kTileHits, kThreadsTile, kTileSmem, s>>>(
-            partials, splits, G, n_pad, n, w.fc1_scale, w.fc1_b, w.fc2_w, w.fc2_b, w.cls_w, w.cls_b, w.mic_w,
-            w.mic_b, dest, debug_logits);
-        return cudaGetLastError();
-    }
-    head_kernel<<<(n + kThreadsHead - 1) / kThreadsHead, kThreadsHead, 0, s>>>(
-        partials, splits, G, n_pad, n, w.fc1_scale, w.fc1_b, w.fc2_w, w.fc2_b, w.cls_w, w.cls_b, w.mic_w, w.mic_b, dest,
-        debug_logits);
-    return cudaGetLastError();
+    if (n > kSmallLaunch)
+        return launch_pdl(head_tile_kernel, dim3((n + kTileHits - 1) / kTileHits), dim3(kThreadsTile), kTileSmem, s,
+                          partials, splits, G, n_pad, n, s1, b1, w2, b2, wc, bc, wm, bm, dest, debug_logits);
+    return launch_pdl(head_kernel, dim3((n + kThreadsHead - 1) / kThreadsHead), dim3(kThreadsHead), 0, s, partials,
+                      splits, G, n_pad, n, s1, b1, w2, b2, wc, bc, wm, bm, dest, debug_logits);
 }
 
 }  // namespace emtk
