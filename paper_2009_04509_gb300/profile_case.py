@@ -1,5 +1,6 @@
 """Profiling driver: a small, self-checking run of the hot path to capture
-with ncu.
+with ncu.  A tool, not part of the library: nothing in the package imports
+it; the commands in profiles/ run it.
 
     python -m paper_2009_04509_gb300.profile_case --mode event   # one APA, 20,000 hits
     python -m paper_2009_04509_gb300.profile_case --mode patches --hits 30000

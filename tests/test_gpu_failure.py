@@ -1,6 +1,6 @@
 """Failure detection without faulting the GPU.
 
-Every mbarrier wait in the tensor-core kernel is bounded by the context's
+Every mbarrier wait in the tensor-core kernels is bounded by the context's
 wait_timeout_ns.  The debug_stall knob makes the kernel wait once on a
 barrier that nothing ever arrives at; the wait must run out, every CTA must
 leave its loops, free its tensor memory and return, and emtk_check must
@@ -27,12 +27,14 @@ def emtk():
     return m
 
 
-def test_bounded_wait_reports_timeout_and_device_stays_usable(emtk):
+@pytest.mark.parametrize("prec", ["bf16", "tf32"])
+def test_bounded_wait_reports_timeout_and_device_stays_usable(emtk, prec):
+    """Both tensor-core kernels: the 16-bit one and the split-fp16 (tf32) one."""
     w = synth.he_normal_weights(0)
     x = synth.inference_patches(300, seed=21) * np.float32(0.05)
     xd = torch.from_numpy(x).cuda()
     scores = torch.zeros((300, 4), device="cuda")
-    stalled = emtk.emtk_create(w, precision="bf16", wait_timeout_ns=50_000_000, debug_stall=True)
+    stalled = emtk.emtk_create(w, precision=prec, wait_timeout_ns=50_000_000, debug_stall=True)
     try:
         emtk.emtk_infer_patches(stalled, xd, scores)
         assert emtk.emtk_check(stalled) == emtk.EMTK_ERR_TIMEOUT
