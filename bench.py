@@ -33,20 +33,26 @@ FLOP_TAIL = 2 * (128 * 32 + 32 * 4)         # 8,448
 FLOP_PER_HIT = FLOP_CONV + FLOP_FC1 + FLOP_TAIL  # 28,444,416
 METRIC = "hit patches/sec on 1 GB300 (extract+CNN); % bf16 tensor peak; gather HBM GB/s"
 
-# DRAM bytes (read + write) of one cnn_tc_kernel launch on the full event, per
+# DRAM bytes (read + write) of one network-kernel launch on the full event, per
 # precision, each from one ncu capture of this benchmark (profiles/launch_list_full_event_*.md),
-# valid for the kernel source they were taken on: reported as null once that source changes.
-TC_TRAFFIC_BYTES = {"bf16": 50_805_504 + 6_386_432, "fp8": 38_858_496 + 1_097_216}
-TC_TRAFFIC_SOURCE_SHA256 = "36b0a0db98821ace"
+# with the kernel source it was taken on: reported as null once that source changes.
+TC_TRAFFIC = {
+    "bf16": (50_887_424 + 6_313_216, "cnn_tc.cu", "1b9fe20a32404eff"),
+    "fp8": (38_884_096 + 1_286_656, "cnn_tc.cu", "1b9fe20a32404eff"),
+    "tf32": (999_452_928 + 403_281_408, "cnn_split.cu", "ba83d319bf0313ba"),
+}
 
 
 def tc_traffic(precision: str, workload: str):
     import hashlib
-    src = os.path.join(ROOT, "paper_2009_04509_gb300", "csrc", "cnn_tc.cu")
-    if precision not in TC_TRAFFIC_BYTES or workload != "full_event" or not os.path.exists(src):
+    if precision not in TC_TRAFFIC or workload != "full_event":
+        return None
+    nbytes, name, sha = TC_TRAFFIC[precision]
+    src = os.path.join(ROOT, "paper_2009_04509_gb300", "csrc", name)
+    if not os.path.exists(src):
         return None
     h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
-    return TC_TRAFFIC_BYTES[precision] if h == TC_TRAFFIC_SOURCE_SHA256 else None
+    return nbytes if h == sha else None
 
 
 def load_peaks():
