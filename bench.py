@@ -549,7 +549,7 @@ def run_service(args, rank, world, local_rank):
 def run_sweep(args, rank, world, local_rank):
     """Inference-only batch sweep: pre-cut fp32 patches (70% zeros, else
     lognormal(2, 1)) through emtk_infer_patches at batch sizes 256 ... 65,536
-    and the paper's 235, 1,693 and 5,358, bf16 and fp32 paths.  Per point:
+    and the paper's 235, 1,693 and 5,358, bf16, fp8, tf32 and fp32 paths.  Per point:
     CUDA events around `steps` calls on the stream, inputs resident, after
     `warmup` calls."""
     import torch
@@ -562,7 +562,7 @@ def run_sweep(args, rank, world, local_rank):
     sc = torch.empty((max(sizes), 4), dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream()
     table = []
-    for prec in ("bf16", "fp8", "fp32"):
+    for prec in ("bf16", "fp8", "tf32", "fp32"):
         ctx = emtk.emtk_create(weights, precision=prec, device=local_rank)
         for n in sizes:
             x = x_all[:n]
@@ -582,11 +582,12 @@ def run_sweep(args, rank, world, local_rank):
         emtk.emtk_destroy(ctx)
     best = max(r["hits_per_s"] for r in table if r["precision"] == "bf16")
     best_fp8 = max(r["hits_per_s"] for r in table if r["precision"] == "fp8")
+    best_tf32 = max(r["hits_per_s"] for r in table if r["precision"] == "tf32")
     out = {"metric": "inference-only batch sweep: patches/s of emtk_infer_patches per batch size", "value": best,
            "unit": "hits/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
            "ms_per_step": None, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-           "dtype": "bf16, fp8 and fp32", "data": "synthetic (pre-cut patches, 70% zeros, lognormal(2,1))",
-           "best_fp8": best_fp8,
+           "dtype": "bf16, fp8, tf32 and fp32", "data": "synthetic (pre-cut patches, 70% zeros, lognormal(2,1))",
+           "best_fp8": best_fp8, "best_tf32": best_tf32,
            "config": {"workload": "pre-cut 48x48 fp32 patches, batch sizes " + ", ".join(map(str, sizes)),
                       "includes": "fp32 -> 16-bit patch conversion (16-bit paths), network, heads"},
            "points": table}
