@@ -297,19 +297,30 @@ def emtk_batcher_create(ctx, nstreams: int = 4, max_hits: int = 65536, max_delay
     return out.value
 
 
+# (batcher, ticket) -> the request's tensors.  The batcher reads and writes them on its
+# own streams after submit returns; holding them here until the ticket is waited for (or
+# the batcher destroyed) keeps torch from freeing and reusing their memory meanwhile.
+_batcher_refs = {}
+
+
 def emtk_batcher_submit(b, adc, nticks: int, hits, scores) -> int:
     """Queues one request (a plane, its hits and its output); returns its ticket.  The tensors
-    must stay alive and unchanged until emtk_batcher_wait has returned for the ticket."""
+    must stay unchanged until emtk_batcher_wait has returned for the ticket; this binding
+    keeps them alive until then."""
     req = make_requests([(adc, nticks, hits, scores)])
     t = ctypes.c_uint64()
     _check(load_library().emtk_batcher_submit(b, req, ctypes.byref(t)), "emtk_batcher_submit")
+    _batcher_refs[(b, t.value)] = (adc, hits, scores)
     return t.value
 
 
 def emtk_batcher_wait(b, ticket: int, timeout_ms: int = -1) -> int:
     """Blocks until the ticket's scores are complete; returns the status (EMTK_ERR_TIMEOUT when
     timeout_ms ran out first, without consuming the ticket)."""
-    return load_library().emtk_batcher_wait(b, int(ticket), int(timeout_ms))
+    rc = load_library().emtk_batcher_wait(b, int(ticket), int(timeout_ms))
+    if rc != EMTK_ERR_TIMEOUT:  # the ticket is done with (or was never issued)
+        _batcher_refs.pop((b, int(ticket)), None)
+    return rc
 
 
 def emtk_batcher_stats(b) -> dict:
@@ -320,6 +331,8 @@ def emtk_batcher_stats(b) -> dict:
 
 def emtk_batcher_destroy(b) -> None:
     _check(load_library().emtk_batcher_destroy(b), "emtk_batcher_destroy")
+    for key in [k for k in _batcher_refs if k[0] == b]:
+        del _batcher_refs[key]
 
 
 # ------------------------------------------------------------- test hooks

@@ -209,3 +209,30 @@ def test_service_configuration(emtk):
         idx = rng.choice(p.nhits, 8, replace=False)
         _, emu = oracle.forward(oracle.extract_patches(p.adc, p.nticks, p.hits[idx]), w, emulate="bf16")
         assert np.abs(got[c][c % 3][idx] - emu).max() <= 2e-2
+
+
+def test_binding_keeps_request_tensors_alive(emtk, planes):
+    """Requests submitted with temporary tensors (no reference kept by the
+    caller): the Python binding holds them until their tickets are waited
+    for, so the batcher never reads memory that torch has freed and reused."""
+    dev = torch.device("cuda:0")
+    w = synth.he_normal_weights(0)
+    ctx = emtk.emtk_create(w, precision="bf16")
+    try:
+        want = direct_scores(emtk, ctx, planes[:3], dev)
+        bat = emtk.emtk_batcher_create(ctx, nstreams=2, max_hits=400, max_delay_us=200)
+        try:
+            outs, tickets = [], []
+            for p in planes[:3]:
+                sc = torch.full((p.nhits, 4), float("nan"), device=dev)
+                tickets.append(emtk.emtk_batcher_submit(bat, torch.from_numpy(p.adc).to(dev), p.nticks,
+                                                        torch.from_numpy(p.hits).to(dev), sc))
+                outs.append(sc)
+            for t in tickets:
+                assert emtk.emtk_batcher_wait(bat, t, 60_000) == emtk.EMTK_OK
+        finally:
+            emtk.emtk_batcher_destroy(bat)
+        for sc, wnt in zip(outs, want):
+            assert np.abs(sc.cpu().numpy() - wnt).max() <= 1e-3
+    finally:
+        emtk.emtk_destroy(ctx)

@@ -139,3 +139,72 @@ def test_tf32_deterministic(emtk, ctx):
     a = run_infer(emtk, ctx, plane.adc, plane.nticks, plane.hits)
     b = run_infer(emtk, ctx, plane.adc, plane.nticks, plane.hits)
     assert np.array_equal(a, b)
+
+
+@pytest.mark.parametrize("scale", [200.0, 0.001])
+def test_tf32_range_ends(emtk, ctx, weights, scale):
+    """The path's range: ADC x 200 puts the largest interval values near 4e4
+    and the largest conv activations near 5e5 (below the 2^20 limit of the
+    head/tail scales); ADC x 0.001 puts most pixel tails in fp16's subnormal
+    range.  Both keep the fp32 bars."""
+    plane = synth.scaled(synth.single_plane(seed=11, nhits=300), scale)
+    got = run_infer(emtk, ctx, plane.adc, plane.nticks, plane.hits)
+    lo, ref = oracle.forward(oracle.extract_patches(plane.adc, plane.nticks, plane.hits), weights)
+    check(got, lo, ref)
+
+
+def test_tf32_chunked_call(emtk, weights):
+    """A context whose workspace holds 256 hits runs a 700-hit call in chunks."""
+    c = emtk.emtk_create(weights, precision="tf32", debug_logits=True, max_hits=256)
+    try:
+        plane = synth.single_plane(seed=10, nhits=700, nticks=1200)
+        got = run_infer(emtk, c, plane.adc, plane.nticks, plane.hits)
+        assert emtk.emtk_get_stats(c)["chunks"] >= 3
+    finally:
+        emtk.emtk_destroy(c)
+    lo, ref = oracle.forward(oracle.extract_patches(plane.adc, plane.nticks, plane.hits), weights)
+    check(got, lo, ref)
+
+
+def test_tf32_batcher_and_host_call(emtk, ctx, weights):
+    """The request batcher and the host-buffer call on a tf32 context: every
+    hit within the fp32 bars of the oracle."""
+    planes = synth.apa(seed=12, hits=(400, 300, 200), n_tracks=6, n_showers=2)
+    want = [oracle.forward(oracle.extract_patches(p.adc, p.nticks, p.hits), weights) for p in planes]
+    b = emtk.emtk_batcher_create(ctx, nstreams=2, max_hits=600, max_delay_us=200)
+    try:
+        outs, tickets, keep = [], [], []
+        for p in planes:
+            # the request's buffers must stay alive until its ticket has been waited for
+            adc, hits = dev(p.adc), dev(p.hits)
+            out = torch.full((p.nhits, 8), float("nan"), device="cuda")
+            keep.append((adc, hits))
+            tickets.append(emtk.emtk_batcher_submit(b, adc, p.nticks, hits, out))
+            outs.append(out)
+        for t in tickets:
+            assert emtk.emtk_batcher_wait(b, t, 60_000) == emtk.EMTK_OK
+    finally:
+        emtk.emtk_batcher_destroy(b)
+    for out, (lo, ref) in zip(outs, want):
+        check(out.cpu().numpy().astype(np.float64), lo, ref)
+    items = [(torch.from_numpy(p.adc).pin_memory(), p.nticks, torch.from_numpy(p.hits).pin_memory(),
+              torch.full((p.nhits, 8), float("nan")).pin_memory()) for p in planes]
+    emtk.emtk_infer_batch_host(ctx, items)
+    torch.cuda.synchronize()
+    assert emtk.emtk_check(ctx) == emtk.EMTK_OK
+    for it, (lo, ref) in zip(items, want):
+        check(it[3].numpy().astype(np.float64), lo, ref)
+
+
+def test_tf32_on_found_hits(emtk, ctx, weights):
+    """Hits found on the plane by emtk_find_hits, scored unchanged."""
+    plane = synth.single_plane(seed=13, nhits=10, nticks=1200)
+    adc = dev(plane.adc)
+    cap = 4096
+    fh = torch.zeros((cap, 2), dtype=torch.int32, device="cuda")
+    n = emtk.emtk_find_hits(ctx, [(adc, plane.nticks, 15.0, fh, None)])[0]
+    assert 0 < n <= cap
+    hits = fh[:n].cpu().numpy()
+    got = run_infer(emtk, ctx, plane.adc, plane.nticks, hits)
+    lo, ref = oracle.forward(oracle.extract_patches(plane.adc, plane.nticks, hits), weights)
+    check(got, lo, ref)
