@@ -529,14 +529,17 @@ emtk_status emtk_infer_patches(emtk_ctx *c, const float *d_patches, int32_t n, f
         const int32_t cnt = (int32_t)std::min<int64_t>(c->max_hits, n - h0);
         const float *src = d_patches + h0 * kPatchElems;
         const void *net_in = src;
-        if (fmt != EMTK_PATCH_F32) {
+        float *rows = d_scores + h0 * out_stride(c);
+        {
+            // the patches in the network's format and each hit's output row, in one launch
             Prof prof(c, EMTK_KERNEL_CONVERT, s);
-            st = cuda_status(launch_convert_patches(src, c->ws.patches, fmt, (int64_t)cnt * kPatchElems, s));
-            net_in = c->ws.patches;
-        }
-        if (st == EMTK_OK) {
-            Prof prof(c, EMTK_KERNEL_CONVERT, s);
-            st = cuda_status(launch_fill_dest(d_scores + h0 * out_stride(c), out_stride(c), c->ws.dest, cnt, s));
+            if (fmt != EMTK_PATCH_F32) {
+                st = cuda_status(launch_convert_patches(src, c->ws.patches, fmt, (int64_t)cnt * kPatchElems, rows,
+                                                        out_stride(c), c->ws.dest, cnt, c->sm_count, s));
+                net_in = c->ws.patches;
+            } else {
+                st = cuda_status(launch_fill_dest(rows, out_stride(c), c->ws.dest, cnt, s));
+            }
         }
         if (st == EMTK_OK) st = run_network(c, net_in, nullptr, cnt, c->ws.dest, s);
     }

@@ -96,7 +96,14 @@ constexpr int kBarAccEmpty = kBarAcc + 1;             // accumulator drained (4 
 constexpr int kBarStall = kBarAccEmpty + 1;
 constexpr int kBarDrain = kBarStall + 1;
 constexpr int kNumBars = kBarDrain + 1;
-constexpr int kOffTmemSlot = kOffBar + kNumBars * 8;
+// accumulator drain: per epilogue warp, 32 rows x 32 outputs staged with a
+// 36-float row pitch (conflict-free 16-byte writes and reads), so each global
+// store of the warp writes four whole 128-byte row pieces
+constexpr int kStagePitch = 36;
+constexpr int kStageBytes = 32 * kStagePitch * 4;  // one epilogue warp
+constexpr int kOffStage = kOffBar + kNumBars * 8 + 8;  // 16-byte aligned below
+constexpr int kOffStageA = (kOffStage + 15) / 16 * 16;
+constexpr int kOffTmemSlot = kOffStageA + 4 * kStageBytes;
 constexpr int kOffAbort = kOffTmemSlot + 4;
 constexpr int kSmemUsed = kOffAbort + 4;
 constexpr int kSmemBytesTC = kSmemUsed + 1024;  // slack for 1024-byte alignment
@@ -144,6 +151,60 @@ __device__ __forceinline__ void load_window_row(const uint16_t *__restrict__ src
     } else {
 #pragma unroll
         for (int j = 0; j < 24; ++j) out[j] = b[j];
+    }
+}
+
+// The first kK rows of a window at once (row r starts at element e0 + r * pitch,
+// pitch a multiple of 8, so every row has the phase e0 % 8): all aligned
+// 16-byte loads are issued before any row is shifted, so the rows cost one
+// round trip to memory instead of kK.
+__device__ __forceinline__ void load_window_rows5(const uint16_t *__restrict__ src, int64_t e0, int64_t pitch,
+                                                  uint32_t (&R)[kK][24]) {
+    const int m = (int)(e0 & 7);
+    uint32_t X[kK][4];  // the seventh chunk of each row (needed when m != 0)
+#pragma unroll
+    for (int r = 0; r < kK; ++r) {
+        const uint4 *p = reinterpret_cast<const uint4 *>(src + (e0 + r * pitch - m));
+#pragma unroll
+        for (int c = 0; c < 6; ++c) {
+            const uint4 v = __ldg(p + c);
+            R[r][4 * c] = v.x;
+            R[r][4 * c + 1] = v.y;
+            R[r][4 * c + 2] = v.z;
+            R[r][4 * c + 3] = v.w;
+        }
+        if (m != 0) {
+            const uint4 v = __ldg(p + 6);
+            X[r][0] = v.x;
+            X[r][1] = v.y;
+            X[r][2] = v.z;
+            X[r][3] = v.w;
+        } else {
+            X[r][0] = X[r][1] = X[r][2] = X[r][3] = 0u;
+        }
+    }
+    if (m == 0) return;
+    const int s = m >> 1;
+#pragma unroll
+    for (int r = 0; r < kK; ++r) {
+        uint32_t w[28];
+#pragma unroll
+        for (int j = 0; j < 24; ++j) w[j] = R[r][j];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) w[24 + j] = X[r][j];
+        uint32_t a[26];
+#pragma unroll
+        for (int j = 0; j < 26; ++j) a[j] = (s & 2) ? w[j + 2] : w[j];
+        uint32_t b[25];
+#pragma unroll
+        for (int j = 0; j < 25; ++j) b[j] = (s & 1) ? a[j + 1] : a[j];
+        if (m & 1) {
+#pragma unroll
+            for (int j = 0; j < 24; ++j) R[r][j] = __funnelshift_r(b[j], b[j + 1], 16);
+        } else {
+#pragma unroll
+            for (int j = 0; j < 24; ++j) R[r][j] = b[j];
+        }
     }
 }
 
@@ -431,16 +492,20 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         };
         // rows y..y+4, slid down one row per y: each window row is loaded once
         uint32_t R[kK][24];
+        if (valid && hd.inside) {
+            load_window_rows5(src, hd.origin + (int64_t)y_first * hd.pitch, hd.pitch, R);
+        } else {
 #pragma unroll
-        for (int i = 0; i < kK - 1; ++i) load_row(y_first + i, R[i]);
+            for (int i = 0; i < kK; ++i) load_row(y_first + i, R[i]);
+        }
         for (int y = y_first; ok && y <= y_last; ++y) {
             if (y > y_first) {
 #pragma unroll
                 for (int i = 0; i < kK - 1; ++i)
 #pragma unroll
                     for (int j = 0; j < 24; ++j) R[i][j] = R[i + 1][j];
+                load_row(y + kK - 1, R[kK - 1]);
             }
-            load_row(y + kK - 1, R[kK - 1]);
 #pragma unroll
             for (int xq = 0; xq < kQ / kPosPerW1; ++xq) {
                 const int quad = (y * kQ) / kPosPerW1 + xq;
@@ -539,22 +604,31 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 tc_fence_after();
                 const int64_t tile = tile0 + tiles_done;
                 const int krow = cta - cta_of_unit(tile * kW1Steps, units, G);
-                const int64_t hit = tile * 128 + row;
-                float *dst = partials + ((int64_t)krow * n_pad + hit) * kN1;
-#pragma unroll
+                // this warp's 32 hits (rows 32 q4 ...) of the tile, 32 outputs at a time
+                const int64_t hit0 = tile * 128 + 32 * q4;
+                float *dst0 = partials + ((int64_t)krow * n_pad + hit0) * kN1;
+                float *stage = reinterpret_cast<float *>(gbase + kOffStageA + q4 * kStageBytes);
+#pragma unroll 1
                 for (int c = 0; c < kN1 / 32; ++c) {
                     uint32_t r[32];
                     tmem_ld16<0>(lane_tmem + kAccCol + 32u * c, r);
                     tmem_ld16<16>(lane_tmem + kAccCol + 32u * c + 16u, r);
                     tmem_ld_wait();
                     reg_fence(r);
-                    if (hit < n) {
 #pragma unroll
-                        for (int e = 0; e < 8; ++e)
-                            reinterpret_cast<float4 *>(dst + 32 * c)[e] =
-                                make_float4(__uint_as_float(r[4 * e]), __uint_as_float(r[4 * e + 1]),
-                                            __uint_as_float(r[4 * e + 2]), __uint_as_float(r[4 * e + 3]));
+                    for (int e = 0; e < 8; ++e)
+                        *reinterpret_cast<uint4 *>(stage + lane * kStagePitch + 4 * e) =
+                            make_uint4(r[4 * e], r[4 * e + 1], r[4 * e + 2], r[4 * e + 3]);
+                    __syncwarp();
+                    // lane l: row 4 k + l / 8, outputs 32 c + 4 (l % 8) ... + 3
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) {
+                        const int i = 4 * k + (lane >> 3);
+                        const float4 v = *reinterpret_cast<const float4 *>(stage + i * kStagePitch + 4 * (lane & 7));
+                        if (hit0 + i < n)
+                            *reinterpret_cast<float4 *>(dst0 + (int64_t)i * kN1 + 32 * c + 4 * (lane & 7)) = v;
                     }
+                    __syncwarp();
                 }
                 tc_fence_before();
                 __syncwarp();

@@ -250,9 +250,11 @@ cudaError_t launch_interval_images(const ReqTable &t, void *dimg, emtk_patch_for
 // Writes patches[(g - g0)] and, if dest != null, dest[g - g0] = output row.
 cudaError_t launch_gather(const ReqTable &t, const void *dimg, emtk_patch_format fmt, int64_t g0,
                           int32_t count, void *patches, float **dest, int out_stride, cudaStream_t s);
-// Patch cut straight from the planes into caller memory (emtk_extract_patches).
-cudaError_t launch_convert_patches(const float *src, void *dst, emtk_patch_format fmt, int64_t n,
-                                   cudaStream_t s);
+// Pre-cut fp32 patches (n values, a multiple of 8, 16-byte aligned) into the
+// network's patch format at dst, and dest[i] = scores + i * out_stride for
+// the nhits hits, in one launch of at most 8 CTAs per SM.
+cudaError_t launch_convert_patches(const float *src, void *dst, emtk_patch_format fmt, int64_t n, float *scores,
+                                   int out_stride, float **dest, int32_t nhits, int sms, cudaStream_t s);
 // Window descriptors of hits [g0, g0+count) (images with halo kHalo), and
 // the output row of each hit in dest.
 cudaError_t launch_hit_desc(const ReqTable &t, int64_t g0, int32_t count, HitDesc *desc, float **dest,
