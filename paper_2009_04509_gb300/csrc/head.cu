@@ -190,28 +190,23 @@ __global__ void __launch_bounds__(kThreadsRows) head_rows_kernel(const float *__
         const int r_end = (int)((int64_t)rows * (share + 1) / kSplit);
         const float4 *p = reinterpret_cast<const float4 *>(partials + h * kN1) + lane;
         float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
-        // this warp's rows in order, loaded 16 at a time so that a hit with many
-        // rows waits for a few round trips, not one per row
+        // this warp's rows in order, loaded kDepth at a time (the last batch
+        // predicated), so that a hit's rows cost one round trip per kDepth rows
         constexpr int kDepth = 16;
-        int r = (int)((int64_t)rows * share / kSplit);
-        for (; r + kDepth <= r_end; r += kDepth) {
+        for (int r = (int)((int64_t)rows * share / kSplit); r < r_end; r += kDepth) {
             float4 v[kDepth];
 #pragma unroll
-            for (int k = 0; k < kDepth; ++k) v[k] = p[(r + k) * row_stride];
+            for (int k = 0; k < kDepth; ++k)
+                if (r + k < r_end) v[k] = p[(r + k) * row_stride];
 #pragma unroll
             for (int k = 0; k < kDepth; ++k) {
-                a.x += v[k].x;
-                a.y += v[k].y;
-                a.z += v[k].z;
-                a.w += v[k].w;
+                if (r + k < r_end) {
+                    a.x += v[k].x;
+                    a.y += v[k].y;
+                    a.z += v[k].z;
+                    a.w += v[k].w;
+                }
             }
-        }
-        for (; r < r_end; ++r) {
-            const float4 v = p[r * row_stride];
-            a.x += v.x;
-            a.y += v.y;
-            a.z += v.z;
-            a.w += v.w;
         }
         if (kSplit > 1) {
             part[jw * 32 + lane] = a;
