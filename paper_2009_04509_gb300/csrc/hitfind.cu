@@ -240,6 +240,7 @@ __global__ void __launch_bounds__(kHfWarps * 32) hf_find_kernel(const __grid_con
                                                                 int32_t *__restrict__ counts,
                                                                 Run *__restrict__ slots) {
     __shared__ float4 stash[kHfWarps][32 * kHfSub];
+    pdl_trigger();  // the place kernel may set up while this one runs; it waits for it
     const int lane = threadIdx.x & 31;
     const int64_t u = (int64_t)blockIdx.x * kHfWarps + (threadIdx.x >> 5);
     if (u >= nunits) return;  // the whole warp leaves together
@@ -275,11 +276,13 @@ __global__ void __launch_bounds__(kHfChunk) hf_place_kernel(const __grid_constan
         const int64_t end = tid + 1 < t.n ? t.r[tid + 1].unit0 : nunits;
         if (t.r[tid].unit0 == end) total[tid] = 0;
     }
-    // the next launch's chunk sums start at zero
+    // the next launch's chunk sums start at zero (this call's find kernel uses the
+    // other array, and the last reader of this one finished before it started)
     for (int64_t i = (int64_t)blockIdx.x * kHfChunk + tid; i < cap; i += (int64_t)gridDim.x * kHfChunk)
         sums_next[i] = 0;
     int r = 0;  // the chunk's plane: the last with chunk0 <= blockIdx.x
     while (r + 1 < t.n && t.r[r + 1].chunk0 <= (int64_t)blockIdx.x) ++r;
+    pdl_wait();  // counts, chunk sums and run slots come from the find kernel
     const HfDesc &d = t.r[r];
     const int64_t pend = r + 1 < t.n ? t.r[r + 1].unit0 : nunits;
     const int64_t c = (int64_t)blockIdx.x - d.chunk0;
@@ -370,9 +373,10 @@ cudaError_t launch_find_hits(const HfTable &t_in, int64_t nunits, void *scratch,
     hf_find_kernel<<<blocks, kHfWarps * 32, 0, s>>>(t, nunits, sums_cur, counts, slots);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    hf_place_kernel<<<(unsigned)nchunks, kHfChunk, 0, s>>>(t, nunits, sums_cur, counts, slots, totals, sums_next,
-                                                            cap);
-    return cudaGetLastError();
+    const int32_t *cc = counts;
+    const Run *cs = slots;
+    return launch_pdl(hf_place_kernel, dim3((unsigned)nchunks), dim3(kHfChunk), 0, s, t, nunits,
+                      static_cast<const int32_t *>(sums_cur), cc, cs, totals, sums_next, cap);
 }
 
 }  // namespace emtk
