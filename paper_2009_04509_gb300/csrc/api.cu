@@ -80,7 +80,7 @@ void free_ctx(emtk_ctx *c) {
         delete[] static_cast<CUtensorMap *>(w.w1_tmap);
     }
     for (void *p : {c->ws.dimg, c->ws.patches, (void *)c->ws.dest, (void *)c->ws.partials, (void *)c->ws.status,
-                    (void *)c->ws.hdesc})
+                    (void *)c->ws.hdesc, (void *)c->ws.tile_done})
         dev_free(p);
     if (c->copy_stream) {
         cudaStreamSynchronize(c->copy_stream);
@@ -195,13 +195,17 @@ emtk_status run_network(emtk_ctx *c, const void *patches, const HitDesc *desc, i
     const int max_splits = (int)std::max<int64_t>(1, kPartialCap / ((int64_t)n_pad * kN1));
     cudaError_t e;
     int splits = 0, G = 0;
+    int *tile_done = nullptr;
     if (tensor_precision(c->opt.precision)) {
         // one persistent CTA per SM (stream-K), fewer if the partial rows would not fit
         G = c->sm_count;
         while (G > 1 && streamk_partial_rows(n, G) > max_splits) G /= 2;
+        // the head of a large launch takes each tile as soon as its partial rows are stored
+        // (16-bit and e4m3 modes; the split-fp16 kernel does not count)
+        if (c->opt.precision != EMTK_TF32 && head_counts_tiles(n, G)) tile_done = c->ws.tile_done;
         Prof prof(c, EMTK_KERNEL_NETWORK, s);
         e = launch_cnn_tc(c->w, patches, desc, tc_mode(c->opt.precision), n, G, c->ws.partials, n_pad,
-                          c->ws.status, c->opt.wait_timeout_ns, c->opt.debug_stall, s);
+                          c->ws.status, c->opt.wait_timeout_ns, c->opt.debug_stall, tile_done, s);
     } else {
         splits = choose_splits_fp32(n, c->sm_count, max_splits);
         Prof prof(c, EMTK_KERNEL_NETWORK, s);
@@ -210,7 +214,8 @@ emtk_status run_network(emtk_ctx *c, const void *patches, const HitDesc *desc, i
     if (e != cudaSuccess) return cuda_status(e);
     {
         Prof prof(c, EMTK_KERNEL_HEAD, s);
-        e = launch_head(c->w, c->ws.partials, splits, G, n_pad, n, dest, c->opt.debug_logits, s);
+        e = launch_head(c->w, c->ws.partials, splits, G, n_pad, n, dest, c->opt.debug_logits, tile_done,
+                        c->ws.status, c->opt.wait_timeout_ns, s);
     }
     count_launch(c, n);
     return cuda_status(e);
@@ -315,6 +320,9 @@ cudaError_t alloc_workspace(emtk_ctx *c, bool patches) {
     }
     if (e == cudaSuccess) e = dmalloc(&c->ws.status, sizeof(int));
     if (e == cudaSuccess) e = cudaMemset(c->ws.status, 0, sizeof(int));
+    const size_t ntiles = (size_t)(o.max_hits + 127) / 128 + 1;
+    if (e == cudaSuccess) e = dmalloc(&c->ws.tile_done, ntiles * sizeof(int));
+    if (e == cudaSuccess) e = cudaMemset(c->ws.tile_done, 0, ntiles * sizeof(int));
     return e;
 }
 
@@ -559,6 +567,9 @@ emtk_status emtk_check(emtk_ctx *c, emtk_stream stream) {
     if (e != cudaSuccess) return EMTK_ERR_CUDA;
     if (status != 0) {
         e = cudaMemset(c->ws.status, 0, sizeof(int));
+        // a launch that gave up may have left tile counters part-way
+        const size_t ntiles = (size_t)(c->opt.max_hits + 127) / 128 + 1;
+        if (e == cudaSuccess && c->ws.tile_done) e = cudaMemset(c->ws.tile_done, 0, ntiles * sizeof(int));
         if (e != cudaSuccess) return EMTK_ERR_CUDA;
         return EMTK_ERR_TIMEOUT;
     }

@@ -231,7 +231,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     cnn_tc_kernel(const __grid_constant__ CUtensorMap tmap_w1, const uint16_t *__restrict__ src,
                   const HitDesc *__restrict__ desc, int n,
                   const uint16_t *__restrict__ convB_g, float *__restrict__ partials, int n_pad, long long units,
-                  int *status, long long timeout_ns, int debug_stall) {
+                  int *status, long long timeout_ns, int debug_stall, int *tile_done) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_u32 = smem_u32(smem_raw);
     const uint32_t base = (raw_u32 + 1023u) & ~1023u;
@@ -543,7 +543,6 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     } else {
         // ================================== conv epilogue + dense-1 store
         const int q4 = warp & 3;
-        const int row = 32 * q4 + lane;
         const uint32_t lane_tmem = tmem + ((uint32_t)(32 * q4) << 16);
         bool ok = true;
         int tiles_done = 0;
@@ -633,6 +632,11 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(bar(kBarAccEmpty));
+                if (tile_done != nullptr) {  // this warp's rows of the tile are stored: count them for the head
+                    __threadfence();
+                    __syncwarp();
+                    if (lane == 0) atomicAdd(tile_done + tile, 1);
+                }
                 ++tiles_done;
             }
         }
@@ -786,7 +790,7 @@ int streamk_partial_rows(int32_t n, int G) {
 
 cudaError_t launch_cnn_tc(const DeviceWeights &w, const void *src, const HitDesc *desc, TcMode mode, int32_t n,
                           int G, float *partials, int n_pad, int *status, int64_t timeout_ns, int debug_stall,
-                          cudaStream_t s) {
+                          int *tile_done, cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
     const CUtensorMap &map = *static_cast<const CUtensorMap *>(w.w1_tmap);
     const long long units = (long long)((n + 127) / 128) * kW1Steps;
@@ -799,7 +803,7 @@ cudaError_t launch_cnn_tc(const DeviceWeights &w, const void *src, const HitDesc
     const uint16_t *convB = w.convB;
     const long long tmo = (long long)timeout_ns;
     return launch_pdl(kernel, grid, dim3(kThreadsTC), kSmemBytesTC, s, map, src16, desc, n, convB, partials, n_pad,
-                      units, status, tmo, debug_stall);
+                      units, status, tmo, debug_stall, tile_done);
 }
 
 }  // namespace emtk

@@ -109,7 +109,8 @@ struct Workspace {
     float **dest = nullptr;      // [max_hits] output row of each hit
     float *partials = nullptr;   // [max_splits][max_hits_pad][128]
     size_t partial_elems = 0;
-    int *status = nullptr;       // device status word (bit 0: a wait gave up)
+    int *status = nullptr;       // device status word (bit 0: a network wait gave up, bit 1: a head wait)
+    int *tile_done = nullptr;    // [max_hits / 128 + 1] per tile: epilogue warps whose partial rows are stored
 };
 
 struct DeviceWeights {
@@ -277,15 +278,24 @@ cudaError_t launch_cnn_fp32(const DeviceWeights &w, const float *patches, int32_
 // = streamk_partial_rows(n, G).
 // src: 16-bit patches [n][48][48] (desc == nullptr) or the haloed interval
 // images of the hits' planes, located through desc.
+// tile_done (or null): each epilogue warp adds 1 to tile_done[tile] once its
+// partial rows of the tile are in memory (a tile is complete at 4 x its
+// partial rows).
 cudaError_t launch_cnn_tc(const DeviceWeights &w, const void *src, const HitDesc *desc, TcMode mode, int32_t n,
                           int G, float *partials, int n_pad, int *status, int64_t timeout_ns, int debug_stall,
-                          cudaStream_t s);
+                          int *tile_done, cudaStream_t s);
 int streamk_partial_rows(int32_t n, int G);
 // Sum of partials + bias + ReLU, dense-2, heads; scores to dest[h].  Partial
 // rows: `splits` per hit (G == 0), or the stream-K contributors of the hit's
-// tile (G > 0).
+// tile (G > 0).  With tile_done (stream-K launches for which
+// head_counts_tiles(n, G) holds), a tile's head starts once the tile's
+// counter is complete instead of after the whole network kernel, gives up
+// when bit 0 of *status is set or after timeout_ns (setting bit 1), and
+// sets the counter back to zero.
+bool head_counts_tiles(int32_t n, int G);
 cudaError_t launch_head(const DeviceWeights &w, const float *partials, int splits, int G, int n_pad,
-                        int32_t n, float *const *dest, int debug_logits, cudaStream_t s);
+                        int32_t n, float *const *dest, int debug_logits, int *tile_done, int *status,
+                        int64_t timeout_ns, cudaStream_t s);
 
 // Kernel attributes (dynamic shared memory), set once per device at create.
 cudaError_t init_fp32_kernel_attrs();

@@ -23,6 +23,12 @@ namespace {
 
 constexpr int kThreadsHead = 128;
 
+__device__ __forceinline__ unsigned long long global_timer() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
 // The dense-2 weights [128][32] into shared memory (16-byte aligned): every
 // load issued before the first store, so that staging costs one round trip.
 template <int kThreads>
@@ -303,13 +309,15 @@ __global__ void __launch_bounds__(kThreadsTile) head_tile_kernel(const float *__
                                                                 const float *__restrict__ cls_b,
                                                                 const float *__restrict__ mic_w,
                                                                 const float *__restrict__ mic_b, float *const *dest,
-                                                                int debug_logits) {
+                                                                int debug_logits, int *tile_done, int *status,
+                                                                long long timeout_ns) {
     extern __shared__ __align__(16) float tsm[];
     float *h1t = tsm;                                    // [kN1][kH1tStride]
     float *w2 = h1t + kN1 * kH1tStride;                  // [kN1][kN2]
     float *h2s = w2 + kN1 * kN2;                         // [kTileHits][kN2 + 1]
     __shared__ __align__(16) float wc[kN2][kNC + 1];
     __shared__ float b2[kN2];
+    __shared__ int go;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     stage_w2<kThreadsTile>(w2, fc2_w);
     for (int i = tid; i < kN2 * kNC; i += kThreadsTile) wc[i / kNC][i % kNC] = cls_w[i];
@@ -317,13 +325,46 @@ __global__ void __launch_bounds__(kThreadsTile) head_tile_kernel(const float *__
         wc[i][kNC] = mic_w[i];
         b2[i] = fc2_b[i];
     }
-    pdl_wait();  // the partial sums and output rows come from the kernels before
     const int64_t h0 = (int64_t)blockIdx.x * kTileHits;
+    const int64_t tile = h0 >> 7;
     int rows = splits;
     if (G > 0) {
         const int64_t units = (int64_t)((n + 127) / 128) * kQuads;
-        const int64_t tile = h0 >> 7;
         rows = cta_of_unit(tile * kQuads + kQuads - 1, units, G) - cta_of_unit(tile * kQuads, units, G) + 1;
+    }
+    if (tile_done != nullptr) {
+        // the tile's partial rows are complete once the 4 epilogue warps of each of its `rows`
+        // CTAs counted theirs; the output rows were written before those CTAs read their
+        // windows.  Every network CTA is running (this kernel is scheduled after all of them
+        // started), so the wait ends unless the network kernel gave up (bit 0 of *status)
+        if (tid == 0) {
+            int ok = 1;
+            const int want = 4 * rows;
+            const long long t0 = (long long)global_timer();
+            for (;;) {
+                int v;
+                asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(tile_done + tile) : "memory");
+                if (v >= want) break;
+                if (*reinterpret_cast<volatile int *>(status) & 1) {
+                    ok = 0;
+                    break;
+                }
+                if ((long long)global_timer() - t0 > timeout_ns) {
+                    atomicOr(status, 2);
+                    ok = 0;
+                    break;
+                }
+                __nanosleep(200);
+            }
+            go = ok;
+        }
+        __syncthreads();
+        if (!go) {
+            if (tid == 0) tile_done[tile] = 0;
+            return;
+        }
+    } else {
+        pdl_wait();  // the partial sums and output rows come from the kernels before
     }
     const int64_t row_stride = (int64_t)n_pad * kN1;  // floats between partial rows
     float bb[4];
@@ -339,7 +380,7 @@ __global__ void __launch_bounds__(kThreadsTile) head_tile_kernel(const float *__
             const int64_t h = h0 + j0 + u * (kThreadsTile / 32);
             const float *p = partials + (h < n ? h : 0) * kN1 + lane;
 #pragma unroll
-            for (int e = 0; e < 4; ++e) a[u][e] = h < n ? p[32 * e] : 0.f;
+            for (int e = 0; e < 4; ++e) a[u][e] = h < n ? __ldcg(p + 32 * e) : 0.f;
         }
         for (int r = 1; r < rows; ++r) {
 #pragma unroll
@@ -347,7 +388,7 @@ __global__ void __launch_bounds__(kThreadsTile) head_tile_kernel(const float *__
                 const int64_t h = h0 + j0 + u * (kThreadsTile / 32);
                 const float *p = partials + (h < n ? h : 0) * kN1 + lane + r * row_stride;
 #pragma unroll
-                for (int e = 0; e < 4; ++e) a[u][e] += h < n ? p[32 * e] : 0.f;
+                for (int e = 0; e < 4; ++e) a[u][e] += h < n ? __ldcg(p + 32 * e) : 0.f;
             }
         }
 #pragma unroll
@@ -357,6 +398,7 @@ __global__ void __launch_bounds__(kThreadsTile) head_tile_kernel(const float *__
                 h1t[(lane + 32 * e) * kH1tStride + j0 + u * (kThreadsTile / 32)] = fmaxf(fmaf(a[u][e], s1, bb[e]), 0.f);
     }
     __syncthreads();
+    if (tile_done != nullptr && tid == 0) tile_done[tile] = 0;  // the tile's rows are read: zero for the next launch
     {
         const int hg = lane, og = warp;  // hits 4hg .. 4hg+3, outputs 4og .. 4og+3
         float acc[4][4];
@@ -398,7 +440,8 @@ __global__ void __launch_bounds__(kThreadsTile) head_tile_kernel(const float *__
     const float m = fmaxf(fmaxf(z[0], z[1]), z[2]);
     const float e0 = expf(z[0] - m), e1 = expf(z[1] - m), e2 = expf(z[2] - m);
     const float sum = e0 + e1 + e2;
-    float *out = dest[h];
+    // through L2: the rows were written by a kernel that is not ordered before this one by its launch
+    float *out = reinterpret_cast<float *>(__ldcg(reinterpret_cast<const unsigned long long *>(dest + h)));
     out[0] = e0 / sum;
     out[1] = e1 / sum;
     out[2] = e2 / sum;
@@ -418,8 +461,13 @@ cudaError_t init_head_kernel_attrs() {
     return cudaFuncSetAttribute(head_tile_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kTileSmem);
 }
 
+bool head_counts_tiles(int32_t n, int G) {
+    return G > 0 && n > kSmallLaunch && streamk_partial_rows(n, G) <= kManyRows;
+}
+
 cudaError_t launch_head(const DeviceWeights &w, const float *partials, int splits, int G, int n_pad, int32_t n,
-                        float *const *dest, int debug_logits, cudaStream_t s) {
+                        float *const *dest, int debug_logits, int *tile_done, int *status, int64_t timeout_ns,
+                        cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
     // most partial rows a hit has: many when a small launch spreads each tile over many CTAs
     const int rows = G > 0 ? streamk_partial_rows(n, G) : splits;
@@ -437,9 +485,12 @@ cudaError_t launch_head(const DeviceWeights &w, const float *partials, int split
         return launch_pdl(head_rows_kernel<32>, dim3((n + 31) / 32), dim3(kThreadsRows), 0, s, partials, splits, G,
                           n_pad, n, s1, b1, w2, b2, wc, bc, wm, bm, dest, debug_logits);
     }
-    if (n > kSmallLaunch)
+    if (n > kSmallLaunch) {
+        const long long tmo = (long long)timeout_ns;
         return launch_pdl(head_tile_kernel, dim3((n + kTileHits - 1) / kTileHits), dim3(kThreadsTile), kTileSmem, s,
-                          partials, splits, G, n_pad, n, s1, b1, w2, b2, wc, bc, wm, bm, dest, debug_logits);
+                          partials, splits, G, n_pad, n, s1, b1, w2, b2, wc, bc, wm, bm, dest, debug_logits,
+                          head_counts_tiles(n, G) ? tile_done : nullptr, status, tmo);
+    }
     return launch_pdl(head_kernel, dim3((n + kThreadsHead - 1) / kThreadsHead), dim3(kThreadsHead), 0, s, partials,
                       splits, G, n_pad, n, s1, b1, w2, b2, wc, bc, wm, bm, dest, debug_logits);
 }

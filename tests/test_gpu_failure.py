@@ -50,3 +50,36 @@ def test_bounded_wait_reports_timeout_and_device_stays_usable(emtk, prec):
         emtk.emtk_destroy(ctx)
     _, emu = oracle.forward(x, w, emulate="bf16")
     assert np.abs(got - emu).max() <= 2e-2
+
+
+def test_bounded_wait_large_launch(emtk):
+    """A launch large enough that each tile's head waits for that tile's
+    counter instead of the whole network kernel (8,192 patches): when the
+    network kernel gives up, the head kernels see its status bit and return
+    at once (no second timeout per tile), emtk_check reports EMTK_ERR_TIMEOUT
+    and clears the status and the tile counters."""
+    import time
+    w = synth.he_normal_weights(0)
+    n = 8192
+    x = synth.inference_patches(n, seed=22) * np.float32(0.05)
+    xd = torch.from_numpy(x).cuda()
+    scores = torch.zeros((n, 4), device="cuda")
+    stalled = emtk.emtk_create(w, precision="bf16", wait_timeout_ns=50_000_000, debug_stall=True)
+    try:
+        t0 = time.perf_counter()
+        emtk.emtk_infer_patches(stalled, xd, scores)
+        assert emtk.emtk_check(stalled) == emtk.EMTK_ERR_TIMEOUT
+        assert time.perf_counter() - t0 < 5.0
+        assert emtk.emtk_check(stalled) == emtk.EMTK_OK
+    finally:
+        emtk.emtk_destroy(stalled)
+    ctx = emtk.emtk_create(w, precision="bf16")
+    try:
+        emtk.emtk_infer_patches(ctx, xd, scores)
+        assert emtk.emtk_check(ctx) == emtk.EMTK_OK
+        got = scores.cpu().numpy().astype(np.float64)
+    finally:
+        emtk.emtk_destroy(ctx)
+    idx = np.arange(0, n, 16)
+    _, emu = oracle.forward(x[idx], w, emulate="bf16")
+    assert np.abs(got[idx] - emu).max() <= 2e-2

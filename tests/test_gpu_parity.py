@@ -283,6 +283,27 @@ def test_deterministic(emtk, ctx_factory, weights):
     assert np.array_equal(a, b)
 
 
+def test_deterministic_large_launch(emtk, ctx_factory, weights):
+    """8,192 pre-cut patches: few partial rows per tile, so each tile's head
+    starts as soon as the tile's rows are stored (per-tile counters, set back
+    to zero by the head).  Three calls in a row on one context give the same
+    bits, and the emulating oracle's scores within the 16-bit bar."""
+    n = 8192
+    x = synth.inference_patches(n, seed=12)
+    xd = torch.from_numpy(x).cuda()
+    ctx = ctx_factory(weights, "bf16")
+    runs = []
+    for _ in range(3):
+        sc = torch.full((n, 8), float("nan"), device="cuda")   # scores, then logits (debug_logits)
+        emtk.emtk_infer_patches(ctx, xd, sc)
+        assert emtk.emtk_check(ctx) == emtk.EMTK_OK
+        runs.append(sc.cpu().numpy())
+    assert np.array_equal(runs[0], runs[1]) and np.array_equal(runs[0], runs[2])
+    idx = np.random.default_rng(0).choice(n, 512, replace=False)
+    _, emu = oracle.forward(x[idx], weights, emulate="bf16")
+    assert np.abs(runs[0][idx, :4].astype(np.float64) - emu).max() <= TOL_16
+
+
 def test_chunked_call_matches(emtk, ctx_factory, weights):
     """A context with a small workspace processes a large call in chunks."""
     plane = synth.single_plane(seed=10, nhits=700, nticks=1200)
