@@ -37,8 +37,8 @@ METRIC = "hit patches/sec on 1 GB300 (extract+CNN); % bf16 tensor peak; gather H
 # precision, each from one ncu capture of this benchmark (profiles/launch_list_full_event_*.md),
 # with the kernel source it was taken on: reported as null once that source changes.
 TC_TRAFFIC = {
-    "bf16": (51_236_608 + 10_781_440, "cnn_tc.cu", "89918cb2f733362b"),
-    "fp8": (38_880_512 + 2_996_992, "cnn_tc.cu", "89918cb2f733362b"),
+    "bf16": (51_318_272 + 9_435_648, "cnn_tc.cu", "1c164a076dd4890c"),
+    "fp8": (38_921_216 + 3_531_520, "cnn_tc.cu", "1c164a076dd4890c"),
     "tf32": (999_452_928 + 403_281_408, "cnn_split.cu", "ba83d319bf0313ba"),
 }
 
