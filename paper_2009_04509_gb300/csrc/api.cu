@@ -88,6 +88,7 @@ void free_ctx(emtk_ctx *c) {
     }
     host_free(c->h_totals);
     dev_free(c->hf_sums);
+    dev_free(c->tile_mask);
     for (auto &st : c->stage) {
         if (st.compute_done) cudaEventSynchronize(st.compute_done);
         dev_free(st.buf);
@@ -251,6 +252,38 @@ void build_table(const emtk_ctx *c, const emtk_request *reqs, int r0, int r1, em
     (void)c;
 }
 
+// Tile-mask geometry of the table's images (bands of kTileRows rows, words of
+// 32 tiles of kTileInts intervals); returns the words of the whole table.
+int64_t assign_tile_masks(ReqTable &t) {
+    int64_t words = 0;
+    for (int i = 0; i < t.n; ++i) {
+        ReqDesc &d = t.r[i];
+        const int64_t rows = d.nwires > 0 ? (int64_t)d.nwires + 2 * d.halo : 0;
+        const int64_t bands = (rows + kTileRows - 1) / kTileRows;
+        const int64_t chunks = ((int64_t)d.pitch + kTileInts - 1) / kTileInts;
+        d.m_wpb = (int32_t)((chunks + 31) / 32);
+        d.m_off = words;
+        words += bands * d.m_wpb;
+    }
+    return words;
+}
+
+// Two zeroed halves of at least `words` mask words each (context field tile_mask).
+emtk_status ensure_tile_masks(emtk_ctx *c, int64_t words, cudaStream_t s) {
+    if (words <= c->tile_mask_cap) return EMTK_OK;
+    cudaError_t e = cudaStreamSynchronize(s);  // earlier launches may still use the old halves
+    if (e == cudaSuccess) e = dev_free(c->tile_mask);
+    c->tile_mask = nullptr;
+    c->tile_mask_cap = 0;
+    const int64_t cap = words + words / 4 + 64;
+    if (e == cudaSuccess) e = dmalloc(&c->tile_mask, 2 * cap * sizeof(uint32_t));
+    if (e == cudaSuccess) e = cudaMemsetAsync(c->tile_mask, 0, 2 * cap * sizeof(uint32_t), s);
+    if (e != cudaSuccess) return cuda_status(e);
+    c->tile_mask_cap = cap;
+    c->tile_mask_parity = 0;
+    return EMTK_OK;
+}
+
 emtk_status run_requests(emtk_ctx *c, const emtk_request *reqs, int32_t nreq, cudaStream_t s) {
     const emtk_patch_format fmt = patch_format(c->opt.precision);
     ReqTable *t = new (std::nothrow) ReqTable;
@@ -268,6 +301,13 @@ emtk_status run_requests(emtk_ctx *c, const emtk_request *reqs, int32_t nreq, cu
             if (t->r[i].nhits == 0) t->r[i].nwires = 0;
         st = ensure_dimg(c, img_bytes, s);
         if (st != EMTK_OK) break;
+        // 16-bit images for the tensor-core kernel: only the tiles some window touches
+        const bool tiles = tc && (fmt == EMTK_PATCH_BF16 || fmt == EMTK_PATCH_F16);
+        const int64_t mask_words = tiles ? assign_tile_masks(*t) : 0;
+        if (tiles) {
+            st = ensure_tile_masks(c, mask_words, s);
+            if (st != EMTK_OK) break;
+        }
         cudaError_t e;
         {
             // the tensor-core kernel reads the windows straight from the images; the
@@ -275,7 +315,17 @@ emtk_status run_requests(emtk_ctx *c, const emtk_request *reqs, int32_t nreq, cu
             const DescJob job{0, (int32_t)std::min<int64_t>(c->max_hits, hits), c->ws.hdesc, c->ws.dest,
                               out_stride(c)};
             Prof prof(c, EMTK_KERNEL_INTERVALS, s);
-            e = launch_interval_images(*t, c->ws.dimg, fmt, s, tc ? &job : nullptr);
+            if (tiles) {
+                uint32_t *cur = c->tile_mask + (int64_t)c->tile_mask_parity * c->tile_mask_cap;
+                uint32_t *next = c->tile_mask + (int64_t)(1 - c->tile_mask_parity) * c->tile_mask_cap;
+                e = launch_cut_tiles(*t, hits, c->ws.dimg, fmt, job, cur, next, c->tile_mask_cap, s);
+                if (e == cudaSuccess)
+                    c->tile_mask_parity ^= 1;
+                else
+                    c->tile_mask_cap = 0;  // the next call reallocates and zeroes both halves
+            } else {
+                e = launch_interval_images(*t, c->ws.dimg, fmt, s, tc ? &job : nullptr);
+            }
         }
         if (e != cudaSuccess) {
             st = cuda_status(e);
@@ -570,6 +620,7 @@ emtk_status emtk_check(emtk_ctx *c, emtk_stream stream) {
         // a launch that gave up may have left tile counters part-way
         const size_t ntiles = (size_t)(c->opt.max_hits + 127) / 128 + 1;
         if (e == cudaSuccess && c->ws.tile_done) e = cudaMemset(c->ws.tile_done, 0, ntiles * sizeof(int));
+        c->tile_mask_cap = 0;  // and tile masks: the next call reallocates and zeroes them
         if (e != cudaSuccess) return EMTK_ERR_CUDA;
         return EMTK_ERR_TIMEOUT;
     }

@@ -55,7 +55,15 @@ struct ReqDesc {
     int32_t pitch;        // row pitch of the interval image (a multiple of 8 elements)
     int32_t halo;         // zero border of the image: element (w, b) is at
                           // d_off + (w + halo) * pitch + (b + halo); rows nwires + 2 halo
+    int32_t m_wpb;        // tile mask (launch_cut_tiles): 32-bit words per band of kTileRows rows
+    int64_t m_off;        // the request's first mask word
 };
+
+// Tiles of an interval image for the cut that skips what no window reads: a
+// tile is kTileRows image rows x kTileInts intervals; tile (band, c) of a
+// request is bit c % 32 of mask word m_off + band * m_wpb + c / 32.
+constexpr int kTileRows = 8;
+constexpr int kTileInts = 32;
 
 // Where the tensor-core kernel finds a hit's 48 x 48 window: element (r, c)
 // is src[origin + r * pitch + c] when `inside` (the whole window lies in the
@@ -213,6 +221,12 @@ struct emtk_ctx {
     int32_t *hf_sums = nullptr;
     int64_t hf_sums_cap = 0;
     int hf_parity = 0;
+    // tiles of the interval images that the hits' windows touch: two zeroed
+    // halves of tile_mask_cap words, used in turn; each tile kernel clears
+    // the other half for the next launch
+    uint32_t *tile_mask = nullptr;
+    int64_t tile_mask_cap = 0;
+    int tile_mask_parity = 0;
 };
 
 namespace emtk {
@@ -247,6 +261,16 @@ struct DescJob {
 };
 cudaError_t launch_interval_images(const ReqTable &t, void *dimg, emtk_patch_format fmt, cudaStream_t s,
                                    const DescJob *job = nullptr);
+// The haloed 16-bit interval images of the table's requests, only the tiles
+// that some hit's window touches (two launches: the hits mark their tiles in
+// mask_cur and the first chunk's window descriptors are built; then one warp
+// per tile computes the covered ones, and mask_next, mask_cap words, is
+// cleared).  Tiles no window touches keep whatever they held: the window
+// reads take their bits only as padding they shift out.  total_hits = all
+// hits of the table.
+cudaError_t launch_cut_tiles(const ReqTable &t, int64_t total_hits, void *dimg, emtk_patch_format fmt,
+                             const DescJob &job, uint32_t *mask_cur, uint32_t *mask_next, int64_t mask_cap,
+                             cudaStream_t s);
 // Patches of hits [g0, g0+count) of the concatenated list (global index).
 // Writes patches[(g - g0)] and, if dest != null, dest[g - g0] = output row.
 cudaError_t launch_gather(const ReqTable &t, const void *dimg, emtk_patch_format fmt, int64_t g0,

@@ -284,6 +284,106 @@ __global__ void __launch_bounds__(256) interval_desc_kernel(const __grid_constan
         hit_desc_one(t, g0, local, desc, dest, out_stride);
 }
 
+// Marks the tiles of request r's image that the window of `hit` touches:
+// image rows [wire, wire + 47] x image columns [bc, bc + 47] (halo 24),
+// clipped to the image.  A hit outside its plane marks the part of its window
+// inside the image (its in-plane pixels are all there).
+__device__ __forceinline__ void mark_window(const ReqDesc &r, const emtk_hit &hit, uint32_t *mask) {
+    const int64_t rows = (int64_t)r.nwires + 2 * r.halo;
+    const int64_t bc = floor_div6(hit.tick);
+    const int64_t r0 = hit.wire > 0 ? hit.wire : 0;
+    const int64_t r1 = (int64_t)hit.wire + 2 * kHalf - 1 < rows - 1 ? (int64_t)hit.wire + 2 * kHalf - 1 : rows - 1;
+    const int64_t c0 = bc > 0 ? bc : 0;
+    const int64_t c1 = bc + 2 * kHalf - 1 < r.pitch - 1 ? bc + 2 * kHalf - 1 : (int64_t)r.pitch - 1;
+    if (r0 > r1 || c0 > c1) return;
+    const int t0 = (int)(c0 / kTileInts), t1 = (int)(c1 / kTileInts);  // at most 3 tiles, at most 2 words
+    for (int64_t band = r0 / kTileRows; band <= r1 / kTileRows; ++band) {
+        uint32_t *row = mask + r.m_off + band * r.m_wpb;
+        for (int wd = t0 >> 5; wd <= (t1 >> 5); ++wd) {
+            const int lo = t0 > 32 * wd ? t0 - 32 * wd : 0;
+            const int hi = t1 < 32 * wd + 31 ? t1 - 32 * wd : 31;
+            const uint32_t bits = (hi == 31 ? 0xffffffffu : ((1u << (hi + 1)) - 1u)) & ~((1u << lo) - 1u);
+            atomicOr(row + wd, bits);
+        }
+    }
+}
+
+// Every hit of the table marks its window's tiles; the first `count` hits from
+// g0 also get their window descriptors and output rows (one thread per hit).
+__global__ void __launch_bounds__(256) mark_desc_kernel(const __grid_constant__ ReqTable t, int64_t total, int64_t g0,
+                                                        int32_t count, HitDesc *desc, float **dest, int out_stride,
+                                                        uint32_t *mask) {
+    pdl_trigger();  // the tile kernel may be scheduled; it waits for this one
+    for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < total;
+         g += (int64_t)gridDim.x * blockDim.x) {
+        const ReqDesc &r = t.r[find_request(t, g)];
+        mark_window(r, r.hits[g - r.hit_begin], mask);
+        if (g >= g0 && g - g0 < count) hit_desc_one(t, g0, g - g0, desc, dest, out_stride);
+    }
+}
+
+// One warp per tile (kTileRows rows x kTileInts intervals = 8 x 16 column
+// pairs) of request blockIdx.y: a tile no window touches is left as it is;
+// the others are computed as in interval_request (same sums, same rounding),
+// four column pairs per lane with every load issued before the first sum.
+// All threads together clear mask_next for the next launch.
+constexpr int kTileWarps = 8;
+template <int FMT>
+__global__ void __launch_bounds__(kTileWarps * 32) interval_tiles_kernel(const __grid_constant__ ReqTable t, void *img,
+                                                                         const uint32_t *mask_cur, uint32_t *mask_next,
+                                                                         int64_t mask_cap) {
+    pdl_trigger();  // the network kernel may set up while this one runs; it waits for it
+    pdl_wait();     // the marks come from the kernel before
+    const int64_t nthr = (int64_t)gridDim.x * gridDim.y * blockDim.x;
+    for (int64_t i = ((int64_t)blockIdx.y * gridDim.x + blockIdx.x) * blockDim.x + threadIdx.x; i < mask_cap;
+         i += nthr)
+        mask_next[i] = 0u;
+    const ReqDesc &r = t.r[blockIdx.y];
+    if (r.nwires == 0) return;
+    const int lane = threadIdx.x & 31;
+    const int rows = r.nwires + 2 * r.halo;
+    const int npairs = r.pitch >> 1;
+    const int nbands = (rows + kTileRows - 1) / kTileRows;
+    const int nchunks = (r.pitch + kTileInts - 1) / kTileInts;
+    const int64_t tile = (int64_t)blockIdx.x * kTileWarps + (threadIdx.x >> 5);
+    if (tile >= (int64_t)nbands * nchunks) return;
+    const int band = (int)(tile / nchunks), chunk = (int)(tile - (int64_t)band * nchunks);
+    if (((mask_cur[r.m_off + (int64_t)band * r.m_wpb + (chunk >> 5)] >> (chunk & 31)) & 1u) == 0) return;
+    constexpr int kPairs = kTileInts / 2;          // column pairs per tile row
+    constexpr int kU = kTileRows * kPairs / 32;    // pairs per lane
+    float4 xa[kU], xd[kU];
+    float2 xb[kU], xc[kU];
+    bool in0[kU], in1[kU];
+    int64_t dst[kU];
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+        const int j = lane + 32 * u;
+        const int wr = band * kTileRows + j / kPairs;
+        const int cp = chunk * kPairs + j % kPairs;
+        const int cb = 2 * cp;
+        const int w = wr - r.halo, b = cb - r.halo;
+        in0[u] = wr < rows && cp < npairs && w >= 0 && w < r.nwires && b >= 0 && b < r.nint;
+        in1[u] = in0[u] && b + 1 < r.nint;
+        dst[u] = (wr < rows && cp < npairs) ? r.d_off + (int64_t)wr * r.pitch + cb : -1;
+        const float *src = r.adc + (int64_t)w * r.ld + 6 * b;
+        if (in0[u]) {
+            xa[u] = __ldcs(reinterpret_cast<const float4 *>(src));
+            xb[u] = __ldcs(reinterpret_cast<const float2 *>(src + 4));
+        }
+        if (in1[u]) {
+            xc[u] = __ldcs(reinterpret_cast<const float2 *>(src + 6));
+            xd[u] = __ldcs(reinterpret_cast<const float4 *>(src + 8));
+        }
+    }
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+        if (dst[u] < 0) continue;
+        const float v0 = in0[u] ? interval_sum(xa[u].x, xa[u].y, xa[u].z, xa[u].w, xb[u].x, xb[u].y) : 0.0f;
+        const float v1 = in1[u] ? interval_sum(xc[u].x, xc[u].y, xd[u].x, xd[u].y, xd[u].z, xd[u].w) : 0.0f;
+        store2<FMT>(img, dst[u], v0, v1, true);
+    }
+}
+
 __global__ void fill_dest_kernel(float *scores, int stride, float **dest, int32_t n) {
     pdl_trigger();
     const int i = blockIdx.x * blockDim.x + threadIdx.x;
@@ -333,6 +433,34 @@ cudaError_t launch_interval_images(const ReqTable &t, void *dimg, emtk_patch_for
     else
         interval_image_kernel<EMTK_PATCH_F16><<<grid, 256, 0, s>>>(t, dimg);
     return cudaGetLastError();
+}
+
+cudaError_t launch_cut_tiles(const ReqTable &t, int64_t total_hits, void *dimg, emtk_patch_format fmt,
+                             const DescJob &job, uint32_t *mask_cur, uint32_t *mask_next, int64_t mask_cap,
+                             cudaStream_t s) {
+    if (total_hits <= 0 || t.n == 0) return cudaSuccess;
+    int64_t mb = (total_hits + 255) / 256;
+    if (mb > 4096) mb = 4096;
+    mark_desc_kernel<<<(unsigned)mb, 256, 0, s>>>(t, total_hits, job.g0, job.count, job.desc, job.dest,
+                                                   job.out_stride, mask_cur);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    int64_t most = 0;  // tiles of the largest image
+    for (int i = 0; i < t.n; ++i) {
+        const ReqDesc &r = t.r[i];
+        if (r.nwires == 0) continue;
+        const int64_t tiles = (((int64_t)r.nwires + 2 * r.halo + kTileRows - 1) / kTileRows) *
+                              ((r.pitch + kTileInts - 1) / kTileInts);
+        most = tiles > most ? tiles : most;
+    }
+    const unsigned bx = (unsigned)((most + kTileWarps - 1) / kTileWarps > 0 ? (most + kTileWarps - 1) / kTileWarps : 1);
+    const dim3 grid(bx, (unsigned)t.n);
+    const uint32_t *mc = mask_cur;
+    if (fmt == EMTK_PATCH_F16)
+        return launch_pdl(interval_tiles_kernel<EMTK_PATCH_F16>, grid, dim3(kTileWarps * 32), 0, s, t, dimg, mc,
+                          mask_next, mask_cap);
+    return launch_pdl(interval_tiles_kernel<EMTK_PATCH_BF16>, grid, dim3(kTileWarps * 32), 0, s, t, dimg, mc,
+                      mask_next, mask_cap);
 }
 
 cudaError_t launch_gather(const ReqTable &t, const void *dimg, emtk_patch_format fmt, int64_t g0, int32_t count,
