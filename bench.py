@@ -424,8 +424,10 @@ def main():
         "extraction": {"bound": "hbm", "achieved": cut_gbs, "peak": peaks["hbm"], "unit": "GB/s",
                        "frac": cut_gbs / peaks["hbm"], "algorithmic_bytes": union + patch_bytes,
                        "bytes_read": union, "bytes_written": patch_bytes,
-                       "kernels": "interval_image_kernel + gather_kernel" if args.precision == "fp32"
-                       else "interval_desc_kernel (images + window descriptors, one launch)",
+                       "kernels": {"fp32": "interval_image_kernel + gather_kernel",
+                                   "tf32": "interval_desc_kernel (images + window descriptors, one launch)"}.get(
+                           args.precision, "mark_tiles_kernel + interval_tiles_kernel (the image tiles some window "
+                                           "touches, and the window descriptors)"),
                        "ms_per_step": cut_ms},
         "step_ms_stats": {"median": statistics.median(step_ms), "min": min(step_ms), "max": max(step_ms),
                           "mean": total_ms / args.steps, "n": len(step_ms)},

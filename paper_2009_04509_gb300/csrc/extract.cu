@@ -284,41 +284,72 @@ __global__ void __launch_bounds__(256) interval_desc_kernel(const __grid_constan
         hit_desc_one(t, g0, local, desc, dest, out_stride);
 }
 
-// Marks the tiles of request r's image that the window of `hit` touches:
-// image rows [wire, wire + 47] x image columns [bc, bc + 47] (halo 24),
-// clipped to the image.  A hit outside its plane marks the part of its window
-// inside the image (its in-plane pixels are all there).
-__device__ __forceinline__ void mark_window(const ReqDesc &r, const emtk_hit &hit, uint32_t *mask) {
+// The tiles of request r's image that the window of `hit` touches: image rows
+// [wire, wire + 47] x image columns [bc, bc + 47] (halo 24), clipped to the
+// image; a hit outside its plane marks the part of its window inside the
+// image (its in-plane pixels are all there).  The window spans at most 7
+// bands and 3 tile columns (2 mask words); `valid` false marks nothing.
+struct WindowTiles {
+    int64_t band0;    // first band
+    int nbands;       // 0 .. 7
+    int w0, nwords;   // first mask word of a band row, 1 or 2
+    uint32_t bits[2]; // tile bits in words w0, w0 + 1
+};
+__device__ __forceinline__ WindowTiles window_tiles(const ReqDesc &r, const emtk_hit &hit, bool valid) {
+    WindowTiles wt{0, 0, 0, 0, {0u, 0u}};
+    if (!valid) return wt;
     const int64_t rows = (int64_t)r.nwires + 2 * r.halo;
     const int64_t bc = floor_div6(hit.tick);
     const int64_t r0 = hit.wire > 0 ? hit.wire : 0;
     const int64_t r1 = (int64_t)hit.wire + 2 * kHalf - 1 < rows - 1 ? (int64_t)hit.wire + 2 * kHalf - 1 : rows - 1;
     const int64_t c0 = bc > 0 ? bc : 0;
     const int64_t c1 = bc + 2 * kHalf - 1 < r.pitch - 1 ? bc + 2 * kHalf - 1 : (int64_t)r.pitch - 1;
-    if (r0 > r1 || c0 > c1) return;
-    const int t0 = (int)(c0 / kTileInts), t1 = (int)(c1 / kTileInts);  // at most 3 tiles, at most 2 words
-    for (int64_t band = r0 / kTileRows; band <= r1 / kTileRows; ++band) {
-        uint32_t *row = mask + r.m_off + band * r.m_wpb;
-        for (int wd = t0 >> 5; wd <= (t1 >> 5); ++wd) {
-            const int lo = t0 > 32 * wd ? t0 - 32 * wd : 0;
-            const int hi = t1 < 32 * wd + 31 ? t1 - 32 * wd : 31;
-            const uint32_t bits = (hi == 31 ? 0xffffffffu : ((1u << (hi + 1)) - 1u)) & ~((1u << lo) - 1u);
-            atomicOr(row + wd, bits);
-        }
+    if (r0 > r1 || c0 > c1) return wt;
+    const int t0 = (int)(c0 / kTileInts), t1 = (int)(c1 / kTileInts);
+    wt.band0 = r0 / kTileRows;
+    wt.nbands = (int)(r1 / kTileRows - wt.band0 + 1);
+    wt.w0 = t0 >> 5;
+    wt.nwords = (t1 >> 5) - wt.w0 + 1;
+    for (int k = 0; k < wt.nwords; ++k) {
+        const int wd = wt.w0 + k;
+        const int lo = t0 > 32 * wd ? t0 - 32 * wd : 0;
+        const int hi = t1 < 32 * wd + 31 ? t1 - 32 * wd : 31;
+        wt.bits[k] = (hi == 31 ? 0xffffffffu : ((1u << (hi + 1)) - 1u)) & ~((1u << lo) - 1u);
     }
+    return wt;
 }
 
-// Every hit of the table marks its window's tiles; the first `count` hits from
-// g0 also get their window descriptors and output rows (one thread per hit).
-__global__ void __launch_bounds__(256) mark_desc_kernel(const __grid_constant__ ReqTable t, int64_t total, int64_t g0,
-                                                        int32_t count, HitDesc *desc, float **dest, int out_stride,
-                                                        uint32_t *mask) {
+// Every hit of request blockIdx.y marks its window's tiles (one thread per
+// hit).  The hits of a block (consecutive in the list: a track or a shower
+// of one plane) mostly mark the same few words, and atomics to one word
+// serialize in L2, so a block first ORs its marks into a shared-memory copy
+// of the plane's mask and then sends each non-zero word once.  A plane whose
+// mask is larger than kMarkSmemWords words marks global memory directly.
+constexpr int kMarkSmemWords = 8192;  // 32 KB
+__global__ void __launch_bounds__(256) mark_tiles_kernel(const __grid_constant__ ReqTable t, uint32_t *mask,
+                                                         int smem_words) {
+    extern __shared__ uint32_t plane_mask[];
     pdl_trigger();  // the tile kernel may be scheduled; it waits for this one
-    for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < total;
-         g += (int64_t)gridDim.x * blockDim.x) {
-        const ReqDesc &r = t.r[find_request(t, g)];
-        mark_window(r, r.hits[g - r.hit_begin], mask);
-        if (g >= g0 && g - g0 < count) hit_desc_one(t, g0, g - g0, desc, dest, out_stride);
+    const ReqDesc &r = t.r[blockIdx.y];
+    const int64_t rows = r.nwires > 0 ? (int64_t)r.nwires + 2 * r.halo : 0;
+    const int64_t words = (rows + kTileRows - 1) / kTileRows * r.m_wpb;
+    const bool local = words <= smem_words;
+    if (local) {
+        for (int64_t i = threadIdx.x; i < words; i += blockDim.x) plane_mask[i] = 0u;
+        __syncthreads();
+    }
+    uint32_t *dst = local ? plane_mask : mask + r.m_off;
+    for (int64_t h = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; h < r.nhits;
+         h += (int64_t)gridDim.x * blockDim.x) {
+        const WindowTiles wt = window_tiles(r, r.hits[h], r.nwires > 0);
+        uint32_t *row0 = dst + wt.band0 * r.m_wpb + wt.w0;
+        for (int b = 0; b < wt.nbands; ++b)
+            for (int k = 0; k < wt.nwords; ++k) atomicOr(row0 + b * r.m_wpb + k, wt.bits[k]);
+    }
+    if (local) {
+        __syncthreads();
+        for (int64_t i = threadIdx.x; i < words; i += blockDim.x)
+            if (plane_mask[i]) atomicOr(mask + r.m_off + i, plane_mask[i]);
     }
 }
 
@@ -326,18 +357,27 @@ __global__ void __launch_bounds__(256) mark_desc_kernel(const __grid_constant__ 
 // pairs) of request blockIdx.y: a tile no window touches is left as it is;
 // the others are computed as in interval_request (same sums, same rounding),
 // four column pairs per lane with every load issued before the first sum.
-// All threads together clear mask_next for the next launch.
+// Grid row blockIdx.y == t.n builds the window descriptors and output rows
+// of hits [g0, g0 + count).  All threads together clear mask_next for the
+// next launch.
 constexpr int kTileWarps = 8;
 template <int FMT>
 __global__ void __launch_bounds__(kTileWarps * 32) interval_tiles_kernel(const __grid_constant__ ReqTable t, void *img,
                                                                          const uint32_t *mask_cur, uint32_t *mask_next,
-                                                                         int64_t mask_cap) {
+                                                                         int64_t mask_cap, int64_t g0, int32_t count,
+                                                                         HitDesc *desc, float **dest, int out_stride) {
     pdl_trigger();  // the network kernel may set up while this one runs; it waits for it
-    pdl_wait();     // the marks come from the kernel before
     const int64_t nthr = (int64_t)gridDim.x * gridDim.y * blockDim.x;
     for (int64_t i = ((int64_t)blockIdx.y * gridDim.x + blockIdx.x) * blockDim.x + threadIdx.x; i < mask_cap;
          i += nthr)
         mask_next[i] = 0u;
+    if ((int)blockIdx.y == t.n) {  // the descriptors need nothing from the marking kernel
+        for (int64_t local = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; local < count;
+             local += (int64_t)gridDim.x * blockDim.x)
+            hit_desc_one(t, g0, local, desc, dest, out_stride);
+        return;
+    }
+    pdl_wait();     // the marks come from the kernel before
     const ReqDesc &r = t.r[blockIdx.y];
     if (r.nwires == 0) return;
     const int lane = threadIdx.x & 31;
@@ -439,10 +479,19 @@ cudaError_t launch_cut_tiles(const ReqTable &t, int64_t total_hits, void *dimg, 
                              const DescJob &job, uint32_t *mask_cur, uint32_t *mask_next, int64_t mask_cap,
                              cudaStream_t s) {
     if (total_hits <= 0 || t.n == 0) return cudaSuccess;
-    int64_t mb = (total_hits + 255) / 256;
+    int64_t most_hits = 0, most_words = 0;
+    for (int i = 0; i < t.n; ++i) {
+        const ReqDesc &r = t.r[i];
+        most_hits = r.nhits > most_hits ? r.nhits : most_hits;
+        const int64_t rows = r.nwires > 0 ? (int64_t)r.nwires + 2 * r.halo : 0;
+        const int64_t words = (rows + kTileRows - 1) / kTileRows * r.m_wpb;
+        most_words = words > most_words ? words : most_words;
+    }
+    int64_t mb = (most_hits + 255) / 256;
     if (mb > 4096) mb = 4096;
-    mark_desc_kernel<<<(unsigned)mb, 256, 0, s>>>(t, total_hits, job.g0, job.count, job.desc, job.dest,
-                                                   job.out_stride, mask_cur);
+    const int smem_words = (int)(most_words < kMarkSmemWords ? most_words : kMarkSmemWords);
+    mark_tiles_kernel<<<dim3((unsigned)(mb > 0 ? mb : 1), (unsigned)t.n), 256, (size_t)smem_words * 4, s>>>(
+        t, mask_cur, smem_words);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     int64_t most = 0;  // tiles of the largest image
@@ -453,14 +502,17 @@ cudaError_t launch_cut_tiles(const ReqTable &t, int64_t total_hits, void *dimg, 
                               ((r.pitch + kTileInts - 1) / kTileInts);
         most = tiles > most ? tiles : most;
     }
-    const unsigned bx = (unsigned)((most + kTileWarps - 1) / kTileWarps > 0 ? (most + kTileWarps - 1) / kTileWarps : 1);
-    const dim3 grid(bx, (unsigned)t.n);
+    int64_t bx = (most + kTileWarps - 1) / kTileWarps;
+    const int64_t desc_blocks = (job.count + kTileWarps * 32 - 1) / (kTileWarps * 32);
+    bx = bx > desc_blocks ? bx : desc_blocks;
+    bx = bx > 0 ? bx : 1;
+    const dim3 grid((unsigned)bx, (unsigned)t.n + 1);  // the last row builds the descriptors
     const uint32_t *mc = mask_cur;
     if (fmt == EMTK_PATCH_F16)
         return launch_pdl(interval_tiles_kernel<EMTK_PATCH_F16>, grid, dim3(kTileWarps * 32), 0, s, t, dimg, mc,
-                          mask_next, mask_cap);
+                          mask_next, mask_cap, job.g0, job.count, job.desc, job.dest, job.out_stride);
     return launch_pdl(interval_tiles_kernel<EMTK_PATCH_BF16>, grid, dim3(kTileWarps * 32), 0, s, t, dimg, mc,
-                      mask_next, mask_cap);
+                      mask_next, mask_cap, job.g0, job.count, job.desc, job.dest, job.out_stride);
 }
 
 cudaError_t launch_gather(const ReqTable &t, const void *dimg, emtk_patch_format fmt, int64_t g0, int32_t count,
