@@ -288,7 +288,8 @@ __global__ void __launch_bounds__(256) interval_desc_kernel(const __grid_constan
 // [wire, wire + 47] x image columns [bc, bc + 47] (halo 24), clipped to the
 // image; a hit outside its plane marks the part of its window inside the
 // image (its in-plane pixels are all there).  The window spans at most 7
-// bands and 3 tile columns (2 mask words); `valid` false marks nothing.
+// bands and 48 / kTileInts + 1 tile columns, in at most 2 mask words;
+// `valid` false marks nothing.
 struct WindowTiles {
     int64_t band0;    // first band
     int nbands;       // 0 .. 7
@@ -353,10 +354,10 @@ __global__ void __launch_bounds__(256) mark_tiles_kernel(const __grid_constant__
     }
 }
 
-// One warp per tile (kTileRows rows x kTileInts intervals = 8 x 16 column
+// One warp per tile (kTileRows rows x kTileInts intervals = 8 x 8 column
 // pairs) of request blockIdx.y: a tile no window touches is left as it is;
 // the others are computed as in interval_request (same sums, same rounding),
-// four column pairs per lane with every load issued before the first sum.
+// two column pairs per lane with every load issued before the first sum.
 // Grid row blockIdx.y == t.n builds the window descriptors and output rows
 // of hits [g0, g0 + count).  All threads together clear mask_next for the
 // next launch.
