@@ -202,8 +202,7 @@ emtk_status run_network(emtk_ctx *c, const void *patches, const HitDesc *desc, i
         G = c->sm_count;
         while (G > 1 && streamk_partial_rows(n, G) > max_splits) G /= 2;
         // the head of a large launch takes each tile as soon as its partial rows are stored
-        // (16-bit and e4m3 modes; the split-fp16 kernel does not count)
-        if (c->opt.precision != EMTK_TF32 && head_counts_tiles(n, G)) tile_done = c->ws.tile_done;
+        if (head_counts_tiles(n, G)) tile_done = c->ws.tile_done;
         Prof prof(c, EMTK_KERNEL_NETWORK, s);
         e = launch_cnn_tc(c->w, patches, desc, tc_mode(c->opt.precision), n, G, c->ws.partials, n_pad,
                           c->ws.status, c->opt.wait_timeout_ns, c->opt.debug_stall, tile_done, s);
@@ -301,8 +300,8 @@ emtk_status run_requests(emtk_ctx *c, const emtk_request *reqs, int32_t nreq, cu
             if (t->r[i].nhits == 0) t->r[i].nwires = 0;
         st = ensure_dimg(c, img_bytes, s);
         if (st != EMTK_OK) break;
-        // 16-bit images for the tensor-core kernel: only the tiles some window touches
-        const bool tiles = tc && (fmt == EMTK_PATCH_BF16 || fmt == EMTK_PATCH_F16);
+        // images for the tensor-core kernels: only the tiles some window touches
+        const bool tiles = tc && (fmt == EMTK_PATCH_BF16 || fmt == EMTK_PATCH_F16 || fmt == kPatchSplit16);
         const int64_t mask_words = tiles ? assign_tile_masks(*t) : 0;
         if (tiles) {
             st = ensure_tile_masks(c, mask_words, s);

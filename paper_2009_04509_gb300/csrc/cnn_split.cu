@@ -138,7 +138,7 @@ __global__ void __launch_bounds__(kThreadsSp, 1)
     cnn_split_kernel(const __grid_constant__ CUtensorMap tmap_hi, const __grid_constant__ CUtensorMap tmap_lo,
                      const uint32_t *__restrict__ src, const HitDesc *__restrict__ desc, int n,
                      const uint16_t *__restrict__ convB_g, float act_mul, float *__restrict__ partials, int n_pad,
-                     long long units, int *status, long long timeout_ns, int debug_stall) {
+                     long long units, int *status, long long timeout_ns, int debug_stall, int *tile_done) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_u32 = smem_u32(smem_raw);
     const uint32_t base = (raw_u32 + 1023u) & ~1023u;
@@ -540,6 +540,12 @@ __global__ void __launch_bounds__(kThreadsSp, 1)
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(bar(kBAccEmpty));
+                // this CTA's last segment of the tile: its partial row is final, count it for the head
+                if (tile_done != nullptr && (pi == np - 1 || pt == kPairsPerTile - 1)) {
+                    __threadfence();
+                    __syncwarp();
+                    if (lane == 0) atomicAdd(tile_done + tile, 1);
+                }
                 ++segs_done;
             }
         }
@@ -659,7 +665,7 @@ cudaError_t prepare_split_weights(DeviceWeights &w, const emtk_weights &hw) {
 
 cudaError_t launch_cnn_split(const DeviceWeights &w, const void *src, const HitDesc *desc, int32_t n, int G,
                              float *partials, int n_pad, int *status, int64_t timeout_ns, int debug_stall,
-                             cudaStream_t s) {
+                             int *tile_done, cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
     const CUtensorMap *maps = static_cast<const CUtensorMap *>(w.w1_tmap);
     const long long units = (long long)((n + 127) / 128) * kQuads;
@@ -668,7 +674,7 @@ cudaError_t launch_cnn_split(const DeviceWeights &w, const void *src, const HitD
     const float act_mul = w.act_mul;
     const long long tmo = (long long)timeout_ns;
     return launch_pdl(cnn_split_kernel, dim3(G), dim3(kThreadsSp), kSmemBytesSp, s, maps[0], maps[1], src32, desc, n,
-                      convB, act_mul, partials, n_pad, units, status, tmo, debug_stall);
+                      convB, act_mul, partials, n_pad, units, status, tmo, debug_stall, tile_done);
 }
 
 }  // namespace emtk

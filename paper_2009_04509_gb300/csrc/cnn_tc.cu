@@ -797,7 +797,7 @@ cudaError_t launch_cnn_tc(const DeviceWeights &w, const void *src, const HitDesc
     const uint16_t *src16 = static_cast<const uint16_t *>(src);
     dim3 grid(G);
     if (mode == kTcSplit)
-        return launch_cnn_split(w, src, desc, n, G, partials, n_pad, status, timeout_ns, debug_stall, s);
+        return launch_cnn_split(w, src, desc, n, G, partials, n_pad, status, timeout_ns, debug_stall, tile_done, s);
     auto *kernel = mode == kTcFp16 ? cnn_tc_kernel<kTcFp16> : mode == kTcFp8 ? cnn_tc_kernel<kTcFp8>
                                                                               : cnn_tc_kernel<kTcBf16>;
     const uint16_t *convB = w.convB;

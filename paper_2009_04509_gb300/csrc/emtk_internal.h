@@ -262,7 +262,8 @@ struct DescJob {
 };
 cudaError_t launch_interval_images(const ReqTable &t, void *dimg, emtk_patch_format fmt, cudaStream_t s,
                                    const DescJob *job = nullptr);
-// The haloed 16-bit interval images of the table's requests, only the tiles
+// The haloed interval images of the table's requests (16-bit, or the split
+// fp16 head / tail words of EMTK_TF32), only the tiles
 // that some hit's window touches (two launches: the hits mark their tiles in
 // mask_cur and the first chunk's window descriptors are built; then one warp
 // per tile computes the covered ones, and mask_next, mask_cap words, is
@@ -333,7 +334,7 @@ cudaError_t prepare_split_weights(DeviceWeights &w, const emtk_weights &hw);
 cudaError_t init_split_kernel_attrs();
 cudaError_t launch_cnn_split(const DeviceWeights &w, const void *src, const HitDesc *desc, int32_t n, int G,
                              float *partials, int n_pad, int *status, int64_t timeout_ns, int debug_stall,
-                             cudaStream_t s);
+                             int *tile_done, cudaStream_t s);
 // EMTK_FP8 weight scale: the largest power of two s_w with max|W1| s_w <= 448.
 double fp8_weight_scale(const float *fc1_w, size_t n);
 int choose_splits_fp32(int n, int sm_count, int max_splits);

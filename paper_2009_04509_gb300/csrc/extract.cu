@@ -509,6 +509,9 @@ cudaError_t launch_cut_tiles(const ReqTable &t, int64_t total_hits, void *dimg, 
     bx = bx > 0 ? bx : 1;
     const dim3 grid((unsigned)bx, (unsigned)t.n + 1);  // the last row builds the descriptors
     const uint32_t *mc = mask_cur;
+    if (fmt == kPatchSplit16)
+        return launch_pdl(interval_tiles_kernel<kPatchSplit16>, grid, dim3(kTileWarps * 32), 0, s, t, dimg, mc,
+                          mask_next, mask_cap, job.g0, job.count, job.desc, job.dest, job.out_stride);
     if (fmt == EMTK_PATCH_F16)
         return launch_pdl(interval_tiles_kernel<EMTK_PATCH_F16>, grid, dim3(kTileWarps * 32), 0, s, t, dimg, mc,
                           mask_next, mask_cap, job.g0, job.count, job.desc, job.dest, job.out_stride);
