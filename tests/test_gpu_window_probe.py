@@ -30,6 +30,16 @@ pixels; the oracle's own fp64 network on the same weights must agree too
 window is probed, through taps that vary over all 25, for hits at every
 phase of the image row (e0 % 8), hits whose window reaches into the zero
 border, hits outside the plane, and, once, through pre-cut patches.
+
+Each probe runs twice: alone (a small launch, whose interval image is built
+from the whole plane) and batched with a 105.6 MB plane holding one hit (a
+launch large enough that only the image tiles some window touches are
+built).  Before the second, two decoy calls on the same context fill the
+image area with other values: one with a plane of another size and row
+pitch, so that most of what becomes the probe image's zero border holds
+data, then one with the probe plane's own layout whose windows rebuild every
+tile that holds probe pixels.  A tile that a window reads but the marking
+missed would then still hold decoy values.
 """
 import numpy as np
 import pytest
@@ -41,6 +51,7 @@ pytestmark = pytest.mark.gpu
 
 NW, NT = 101, 2399          # 399 complete intervals and a partial one (5 ticks)
 NINT = NT // 6
+BIG_NW, BIG_NT = 4400, 6000  # 105.6 MB of ADC: a launch holding it cuts only the touched image tiles
 
 
 @pytest.fixture(scope="module")
@@ -53,8 +64,15 @@ def emtk():
     return m
 
 
-def probe_plane():
-    rng = np.random.default_rng(77)
+@pytest.fixture(scope="module")
+def big(emtk):
+    adc = torch.zeros((BIG_NW, BIG_NT), dtype=torch.float32, device="cuda")
+    hits = torch.tensor([[BIG_NW // 2, BIG_NT // 2]], dtype=torch.int32, device="cuda")
+    return adc, hits
+
+
+def probe_plane(seed=77):
+    rng = np.random.default_rng(seed)
     v = rng.integers(0, 16, (NW, NINT)).astype(np.float32)
     a = rng.integers(0, 4, (NW, NINT)).astype(np.float32)
     b = rng.integers(0, 4, (NW, NINT)).astype(np.float32)
@@ -78,6 +96,24 @@ def probe_hits():
     h = np.array(h, np.int32)
     reps = -(-150 // len(h))
     return np.concatenate([h] * reps)[:150]   # two 128-hit tiles, the second ragged
+
+
+DA_NW, DA_NT, DA_LD = NW + 48, NT + 240, 2644   # the first decoy's plane: other rows, other pitch
+
+
+def decoy_a():
+    """A plane of another shape and windows covering all of its image."""
+    adc = np.random.default_rng(79).integers(1, 16, (DA_NW, DA_LD)).astype(np.float32)
+    hits = [[w, 6 * b + 3] for w in range(0, DA_NW + 48, 40) for b in range(0, DA_NT // 6 + 48, 40)]
+    return adc, np.array(hits, np.int32)
+
+
+def decoy_b_hits():
+    """Windows of in-plane hits covering every image tile that holds probe
+    pixels (wires 0..NW-1, intervals 0..NINT-1) and fewer of the border tiles."""
+    ws = [24, 64, NW - 24]
+    bs = list(range(24, NINT - 24, 40)) + [NINT - 24]
+    return np.array([[w, 6 * b + 3] for w in ws for b in bs], np.int32)
 
 
 def probe_pixels(per_logit):
@@ -127,7 +163,7 @@ def expected_logits(patches, where, n):
 
 
 @pytest.mark.parametrize("prec", ["bf16", "fp16", "fp8", "tf32"])
-def test_window_read_bit_exact(emtk, prec):
+def test_window_read_bit_exact(emtk, big, prec):
     adc_np, _ = probe_plane()
     hits_np = probe_hits()
     n = hits_np.shape[0]
@@ -137,6 +173,15 @@ def test_window_read_bit_exact(emtk, prec):
     adc = torch.from_numpy(adc_np).cuda()
     hits = torch.from_numpy(hits_np).cuda()
     patches = torch.from_numpy(want_p).cuda()
+    da_np, da_hits_np = decoy_a()
+    da, da_hits = torch.from_numpy(da_np).cuda(), torch.from_numpy(da_hits_np).cuda()
+    db_np, _ = probe_plane(seed=78)
+    assert (db_np[:, :NINT * 6] != adc_np[:, :NINT * 6]).any()
+    db, db_hits = torch.from_numpy(db_np).cuda(), torch.from_numpy(decoy_b_hits()).cuda()
+    big_adc, big_hits = big
+    big_out = torch.empty((1, 8), dtype=torch.float32, device="cuda")
+    da_out = torch.empty((da_hits.shape[0], 8), dtype=torch.float32, device="cuda")
+    db_out = torch.empty((db_hits.shape[0], 8), dtype=torch.float32, device="cuda")
     per_logit = 3 if prec == "fp8" else 6
     groups = probe_pixels(per_logit)
     if prec in ("fp16", "fp8"):
@@ -147,6 +192,10 @@ def test_window_read_bit_exact(emtk, prec):
         try:
             out = torch.full((n, 8), float("nan"), dtype=torch.float32, device="cuda")
             emtk.emtk_infer(ctx, adc, NT, hits, out)
+            emtk.emtk_infer_batch(ctx, [(da, DA_NT, da_hits, da_out), (big_adc, BIG_NT, big_hits, big_out)])
+            emtk.emtk_infer_batch(ctx, [(db, NT, db_hits, db_out), (big_adc, BIG_NT, big_hits, big_out)])
+            tiled = torch.full((n, 8), float("nan"), dtype=torch.float32, device="cuda")
+            emtk.emtk_infer_batch(ctx, [(adc, NT, hits, tiled), (big_adc, BIG_NT, big_hits, big_out)])
             via_patches = None
             if gi == 0:                    # the pre-cut patch path reads the same windows
                 via_patches = torch.full((n, 8), float("nan"), dtype=torch.float32, device="cuda")
@@ -159,6 +208,11 @@ def test_window_read_bit_exact(emtk, prec):
         bad = np.argwhere(got != want)
         assert bad.size == 0, (f"{prec}, pixel group {gi}: {len(bad)} logits differ, first at hit "
                                f"{hits_np[bad[0][0]].tolist()} logit {bad[0][1]}: {got[tuple(bad[0])]} "
+                               f"!= {want[tuple(bad[0])]}")
+        got_t = tiled[:, 4:].cpu().numpy().astype(np.float64)
+        bad = np.argwhere(got_t != want)
+        assert bad.size == 0, (f"{prec}, tiled cut, pixel group {gi}: {len(bad)} logits differ, first at hit "
+                               f"{hits_np[bad[0][0]].tolist()} logit {bad[0][1]}: {got_t[tuple(bad[0])]} "
                                f"!= {want[tuple(bad[0])]}")
         if via_patches is not None:
             assert np.array_equal(via_patches[:, 4:].cpu().numpy().astype(np.float64), want)
