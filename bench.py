@@ -647,7 +647,8 @@ def run_sweep(args, rank, world, local_rank):
            "dtype": "bf16, fp8, tf32 and fp32", "data": "synthetic (pre-cut patches, 70% zeros, lognormal(2,1))",
            "best_fp8": best_fp8, "best_tf32": best_tf32,
            "config": {"workload": "pre-cut 48x48 fp32 patches, batch sizes " + ", ".join(map(str, sizes)),
-                      "includes": "fp32 -> 16-bit patch conversion (16-bit paths), network, heads"},
+                      "includes": "network (the 16-bit and fp8 kernels read the fp32 patches and round them as they "
+                                  "load them; tf32: a conversion launch to split-fp16 words first), heads"},
            "points": table}
     if rank == 0:
         print(json.dumps(out))

@@ -149,7 +149,7 @@ typedef enum {
     EMTK_KERNEL_GATHER = 1,    /* interval image -> 48x48 patches */
     EMTK_KERNEL_NETWORK = 2,   /* conv + dense-1 (tensor cores or fp32) */
     EMTK_KERNEL_HEAD = 3,      /* dense-1 sum + dense-2 + heads */
-    EMTK_KERNEL_CONVERT = 4,   /* fp32 patches -> 16 bit (emtk_infer_patches) */
+    EMTK_KERNEL_CONVERT = 4,   /* fp32 patches -> split-fp16 words (emtk_infer_patches, EMTK_TF32) */
     EMTK_KERNEL_HITFIND = 5,   /* hit finding (emtk_find_hits: find, place) */
     EMTK_NUM_KERNELS = 6
 } emtk_kernel;
@@ -247,7 +247,11 @@ EMTK_API emtk_status emtk_extract_patches_static(const float *d_adc, int32_t nwi
                                                  const emtk_hit *d_hits, int32_t nhits, void *d_patches,
                                                  emtk_patch_format fmt, emtk_stream stream);
 
-/* Network only (Sec. 2.2) on pre-cut fp32 patches [n][48][48] -> d_scores. */
+/* Network only (Sec. 2.2) on pre-cut fp32 patches [n][48][48] -> d_scores.
+ * The 16-bit and fp8 network kernels read the fp32 patches themselves, each
+ * value rounded to nearest-even 16 bit as it is loaded; EMTK_TF32 converts
+ * them to head/tail words in one launch first.  d_patches 16-byte aligned,
+ * d_scores 4-byte aligned; chunks of max_hits patches per launch. */
 EMTK_API emtk_status emtk_infer_patches(emtk_ctx *ctx, const float *d_patches, int32_t n, float *d_scores,
                                emtk_stream stream);
 

@@ -189,8 +189,8 @@ emtk_status ensure_dimg(emtk_ctx *c, size_t bytes, cudaStream_t s) {
 // Network on `n` patches already in the workspace format -> scores via dest.
 // `desc` (tensor-core path only) locates each hit's window in the haloed
 // interval images at `patches`; without it `patches` holds the patches.
-emtk_status run_network(emtk_ctx *c, const void *patches, const HitDesc *desc, int32_t n, float *const *dest,
-                        cudaStream_t s) {
+emtk_status run_network(emtk_ctx *c, const void *patches, const HitDesc *desc, int32_t n, OutRows out_rows,
+                        const float *src32, cudaStream_t s) {
     if (n <= 0) return EMTK_OK;
     const int n_pad = n_pad_of(n);
     const int max_splits = (int)std::max<int64_t>(1, kPartialCap / ((int64_t)n_pad * kN1));
@@ -205,7 +205,7 @@ emtk_status run_network(emtk_ctx *c, const void *patches, const HitDesc *desc, i
         if (head_counts_tiles(n, G)) tile_done = c->ws.tile_done;
         Prof prof(c, EMTK_KERNEL_NETWORK, s);
         e = launch_cnn_tc(c->w, patches, desc, tc_mode(c->opt.precision), n, G, c->ws.partials, n_pad,
-                          c->ws.status, c->opt.wait_timeout_ns, c->opt.debug_stall, tile_done, s);
+                          c->ws.status, c->opt.wait_timeout_ns, c->opt.debug_stall, tile_done, src32, s);
     } else {
         splits = choose_splits_fp32(n, c->sm_count, max_splits);
         Prof prof(c, EMTK_KERNEL_NETWORK, s);
@@ -214,7 +214,7 @@ emtk_status run_network(emtk_ctx *c, const void *patches, const HitDesc *desc, i
     if (e != cudaSuccess) return cuda_status(e);
     {
         Prof prof(c, EMTK_KERNEL_HEAD, s);
-        e = launch_head(c->w, c->ws.partials, splits, G, n_pad, n, dest, c->opt.debug_logits, tile_done,
+        e = launch_head(c->w, c->ws.partials, splits, G, n_pad, n, out_rows, c->opt.debug_logits, tile_done,
                         c->ws.status, c->opt.wait_timeout_ns, s);
     }
     count_launch(c, n);
@@ -353,8 +353,9 @@ emtk_status run_requests(emtk_ctx *c, const emtk_request *reqs, int32_t nreq, cu
                 st = cuda_status(e);
                 break;
             }
-            st = tc ? run_network(c, c->ws.dimg, c->ws.hdesc, cnt, c->ws.dest, s)
-                    : run_network(c, c->ws.patches, nullptr, cnt, c->ws.dest, s);
+            const OutRows out{c->ws.dest, nullptr, 0};
+            st = tc ? run_network(c, c->ws.dimg, c->ws.hdesc, cnt, out, nullptr, s)
+                    : run_network(c, c->ws.patches, nullptr, cnt, out, nullptr, s);
         }
         c->stats.hits += hits;
     }
@@ -368,7 +369,8 @@ cudaError_t alloc_workspace(emtk_ctx *c, bool patches) {
     const emtk_options &o = c->opt;
     const emtk_patch_format fmt = patch_format(o.precision);
     cudaError_t e = cudaSuccess;
-    if (patches || !tensor_precision(o.precision))
+    // the 16-bit and fp8 tensor-core kernels read pre-cut fp32 patches themselves
+    if ((patches && fmt == kPatchSplit16) || !tensor_precision(o.precision))
         e = dmalloc(&c->ws.patches, (size_t)o.max_hits * kPatchElems * patch_elem_bytes(fmt));
     if (e == cudaSuccess) e = dmalloc(&c->ws.dest, (size_t)o.max_hits * sizeof(float *));
     if (e == cudaSuccess && tensor_precision(o.precision))
@@ -597,6 +599,12 @@ emtk_status emtk_infer_patches(emtk_ctx *c, const float *d_patches, int32_t n, f
         const float *src = d_patches + h0 * kPatchElems;
         const void *net_in = src;
         float *rows = d_scores + h0 * out_stride(c);
+        if (fmt == EMTK_PATCH_BF16 || fmt == EMTK_PATCH_F16) {
+            // the tensor-core kernel reads the fp32 patches itself (no conversion launch), and
+            // the head writes each hit's scores to rows + h * stride
+            st = run_network(c, nullptr, nullptr, cnt, OutRows{nullptr, rows, out_stride(c)}, src, s);
+            continue;
+        }
         {
             // the patches in the network's format and each hit's output row, in one launch
             Prof prof(c, EMTK_KERNEL_CONVERT, s);
@@ -608,7 +616,7 @@ emtk_status emtk_infer_patches(emtk_ctx *c, const float *d_patches, int32_t n, f
                 st = cuda_status(launch_fill_dest(rows, out_stride(c), c->ws.dest, cnt, s));
             }
         }
-        if (st == EMTK_OK) st = run_network(c, net_in, nullptr, cnt, c->ws.dest, s);
+        if (st == EMTK_OK) st = run_network(c, net_in, nullptr, cnt, OutRows{c->ws.dest, nullptr, 0}, nullptr, s);
     }
     c->stats.calls++;
     c->stats.hits += (uint64_t)n;

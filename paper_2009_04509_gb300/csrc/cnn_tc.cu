@@ -208,6 +208,33 @@ __device__ __forceinline__ void load_window_rows5(const uint16_t *__restrict__ s
     }
 }
 
+// Two fp32 values rounded to nearest-even 16 bit (bf16, or fp16 if FP16) and
+// packed, the first in the low half: the rounding of the patch conversion.
+template <bool FP16>
+__device__ __forceinline__ uint32_t pack_rn16(float lo, float hi) {
+    if (FP16) {
+        const __half2 h = __floats2half2_rn(lo, hi);
+        return *reinterpret_cast<const uint32_t *>(&h);
+    }
+    const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<const uint32_t *>(&h);
+}
+
+// One 48-value row of a pre-cut fp32 patch (element e0 of src, 16-byte
+// aligned): twelve 16-byte loads, rounded to 16 bit, two pixels per word.
+template <bool FP16>
+__device__ __forceinline__ void load_patch_row_f32(const float *__restrict__ src, int64_t e0, uint32_t (&out)[24]) {
+    const float4 *p = reinterpret_cast<const float4 *>(src + e0);
+    float4 v[12];
+#pragma unroll
+    for (int c = 0; c < 12; ++c) v[c] = __ldg(p + c);
+#pragma unroll
+    for (int c = 0; c < 12; ++c) {
+        out[2 * c] = pack_rn16<FP16>(v[c].x, v[c].y);
+        out[2 * c + 1] = pack_rn16<FP16>(v[c].z, v[c].w);
+    }
+}
+
 // The same row for a hit whose window leaves the haloed image (a hit outside
 // its plane): every pixel checked against the plane, zero outside.
 __device__ __forceinline__ void load_window_row_checked(const uint16_t *__restrict__ src, const HitDesc &hd, int r,
@@ -231,7 +258,8 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     cnn_tc_kernel(const __grid_constant__ CUtensorMap tmap_w1, const uint16_t *__restrict__ src,
                   const HitDesc *__restrict__ desc, int n,
                   const uint16_t *__restrict__ convB_g, float *__restrict__ partials, int n_pad, long long units,
-                  int *status, long long timeout_ns, int debug_stall, int *tile_done) {
+                  int *status, long long timeout_ns, int debug_stall, int *tile_done,
+                  const float *__restrict__ src32) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_u32 = smem_u32(smem_raw);
     const uint32_t base = (raw_u32 + 1023u) & ~1023u;
@@ -484,6 +512,8 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
             if (!valid) {
 #pragma unroll
                 for (int j = 0; j < 24; ++j) out[j] = 0u;
+            } else if (src32 != nullptr) {
+                load_patch_row_f32<FP16>(src32, hd.origin + (int64_t)r * kPatch, out);
             } else if (hd.inside) {
                 load_window_row(src, hd.origin + (int64_t)r * hd.pitch, out);
             } else {
@@ -492,7 +522,7 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         };
         // rows y..y+4, slid down one row per y: each window row is loaded once
         uint32_t R[kK][24];
-        if (valid && hd.inside) {
+        if (valid && hd.inside && src32 == nullptr) {
             load_window_rows5(src, hd.origin + (int64_t)y_first * hd.pitch, hd.pitch, R);
         } else {
 #pragma unroll
@@ -790,7 +820,7 @@ int streamk_partial_rows(int32_t n, int G) {
 
 cudaError_t launch_cnn_tc(const DeviceWeights &w, const void *src, const HitDesc *desc, TcMode mode, int32_t n,
                           int G, float *partials, int n_pad, int *status, int64_t timeout_ns, int debug_stall,
-                          int *tile_done, cudaStream_t s) {
+                          int *tile_done, const float *src32, cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
     const CUtensorMap &map = *static_cast<const CUtensorMap *>(w.w1_tmap);
     const long long units = (long long)((n + 127) / 128) * kW1Steps;
@@ -803,7 +833,7 @@ cudaError_t launch_cnn_tc(const DeviceWeights &w, const void *src, const HitDesc
     const uint16_t *convB = w.convB;
     const long long tmo = (long long)timeout_ns;
     return launch_pdl(kernel, grid, dim3(kThreadsTC), kSmemBytesTC, s, map, src16, desc, n, convB, partials, n_pad,
-                      units, status, tmo, debug_stall, tile_done);
+                      units, status, tmo, debug_stall, tile_done, src32);
 }
 
 }  // namespace emtk

@@ -307,11 +307,21 @@ cudaError_t launch_cnn_fp32(const DeviceWeights &w, const float *patches, int32_
 // tile_done (or null): each epilogue warp adds 1 to tile_done[tile] once its
 // partial rows of the tile are in memory (a tile is complete at 4 x its
 // partial rows).
+// src32 (or null; 16-bit and fp8 modes, desc == nullptr): pre-cut fp32
+// patches [n][48][48] that the kernel reads itself, rounding each value as the
+// patch conversion does.
 cudaError_t launch_cnn_tc(const DeviceWeights &w, const void *src, const HitDesc *desc, TcMode mode, int32_t n,
                           int G, float *partials, int n_pad, int *status, int64_t timeout_ns, int debug_stall,
-                          int *tile_done, cudaStream_t s);
+                          int *tile_done, const float *src32, cudaStream_t s);
+// Where the head writes hit h's scores: dest[h], or rows + h * stride when
+// rows is not null (pre-cut patches, whose rows are consecutive).
+struct OutRows {
+    float *const *dest;
+    float *rows;
+    int stride;
+};
 int streamk_partial_rows(int32_t n, int G);
-// Sum of partials + bias + ReLU, dense-2, heads; scores to dest[h].  Partial
+// Sum of partials + bias + ReLU, dense-2, heads; hit h's scores where out_rows says.  Partial
 // rows: `splits` per hit (G == 0), or the stream-K contributors of the hit's
 // tile (G > 0).  With tile_done (stream-K launches for which
 // head_counts_tiles(n, G) holds), a tile's head starts once the tile's
@@ -320,7 +330,7 @@ int streamk_partial_rows(int32_t n, int G);
 // sets the counter back to zero.
 bool head_counts_tiles(int32_t n, int G);
 cudaError_t launch_head(const DeviceWeights &w, const float *partials, int splits, int G, int n_pad,
-                        int32_t n, float *const *dest, int debug_logits, int *tile_done, int *status,
+                        int32_t n, OutRows out_rows, int debug_logits, int *tile_done, int *status,
                         int64_t timeout_ns, cudaStream_t s);
 
 // Kernel attributes (dynamic shared memory), set once per device at create.

@@ -53,7 +53,7 @@ __global__ void __launch_bounds__(kThreadsHead) head_kernel(const float *__restr
                                                            const float *__restrict__ cls_w,
                                                            const float *__restrict__ cls_b,
                                                            const float *__restrict__ mic_w,
-                                                           const float *__restrict__ mic_b, float *const *dest,
+                                                           const float *__restrict__ mic_b, OutRows out_rows,
                                                            int debug_logits) {
     __shared__ __align__(16) float w2[kN1][kN2];
     __shared__ __align__(16) float wc[kN2][kNC + 1];
@@ -123,7 +123,7 @@ __global__ void __launch_bounds__(kThreadsHead) head_kernel(const float *__restr
     const float m = fmaxf(fmaxf(z[0], z[1]), z[2]);
     const float e0 = expf(z[0] - m), e1 = expf(z[1] - m), e2 = expf(z[2] - m);
     const float sum = e0 + e1 + e2;
-    float *out = dest[h];
+    float *out = out_rows.rows ? out_rows.rows + h * (int64_t)out_rows.stride : out_rows.dest[h];
     out[0] = e0 / sum;
     out[1] = e1 / sum;
     out[2] = e2 / sum;
@@ -160,7 +160,7 @@ __global__ void __launch_bounds__(kThreadsRows) head_rows_kernel(const float *__
                                                                 const float *__restrict__ cls_w,
                                                                 const float *__restrict__ cls_b,
                                                                 const float *__restrict__ mic_w,
-                                                                const float *__restrict__ mic_b, float *const *dest,
+                                                                const float *__restrict__ mic_b, OutRows out_rows,
                                                                 int debug_logits) {
     static_assert(kHitsRows * kSplit <= kThreadsRows / 32 || kSplit == 1, "a warp per (hit, row share)");
     __shared__ float h1s[kHitsRows * kH1Stride];
@@ -272,7 +272,7 @@ __global__ void __launch_bounds__(kThreadsRows) head_rows_kernel(const float *__
     const float m = fmaxf(fmaxf(z[0], z[1]), z[2]);
     const float e0 = expf(z[0] - m), e1 = expf(z[1] - m), e2 = expf(z[2] - m);
     const float sum = e0 + e1 + e2;
-    float *out = dest[h];
+    float *out = out_rows.rows ? out_rows.rows + h * (int64_t)out_rows.stride : out_rows.dest[h];
     out[0] = e0 / sum;
     out[1] = e1 / sum;
     out[2] = e2 / sum;
@@ -308,7 +308,7 @@ __global__ void __launch_bounds__(kThreadsTile) head_tile_kernel(const float *__
                                                                 const float *__restrict__ cls_w,
                                                                 const float *__restrict__ cls_b,
                                                                 const float *__restrict__ mic_w,
-                                                                const float *__restrict__ mic_b, float *const *dest,
+                                                                const float *__restrict__ mic_b, OutRows out_rows,
                                                                 int debug_logits, int *tile_done, int *status,
                                                                 long long timeout_ns) {
     extern __shared__ __align__(16) float tsm[];
@@ -441,7 +441,9 @@ __global__ void __launch_bounds__(kThreadsTile) head_tile_kernel(const float *__
     const float e0 = expf(z[0] - m), e1 = expf(z[1] - m), e2 = expf(z[2] - m);
     const float sum = e0 + e1 + e2;
     // through L2: the rows were written by a kernel that is not ordered before this one by its launch
-    float *out = reinterpret_cast<float *>(__ldcg(reinterpret_cast<const unsigned long long *>(dest + h)));
+    float *out = out_rows.rows ? out_rows.rows + h * (int64_t)out_rows.stride
+                               : reinterpret_cast<float *>(
+                                     __ldcg(reinterpret_cast<const unsigned long long *>(out_rows.dest + h)));
     out[0] = e0 / sum;
     out[1] = e1 / sum;
     out[2] = e2 / sum;
@@ -466,7 +468,7 @@ bool head_counts_tiles(int32_t n, int G) {
 }
 
 cudaError_t launch_head(const DeviceWeights &w, const float *partials, int splits, int G, int n_pad, int32_t n,
-                        float *const *dest, int debug_logits, int *tile_done, int *status, int64_t timeout_ns,
+                        OutRows out_rows, int debug_logits, int *tile_done, int *status, int64_t timeout_ns,
                         cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
     // most partial rows a hit has: many when a small launch spreads each tile over many CTAs
@@ -478,21 +480,21 @@ cudaError_t launch_head(const DeviceWeights &w, const float *partials, int split
     if (rows > kManyRows) {
         if (rows >= kSplitRows && n <= kSmallLaunch)  // a hit's rows over 4 warps, 2 hits per block
             return launch_pdl(head_rows_kernel<2, 4>, dim3((n + 1) / 2), dim3(kThreadsRows), 0, s, partials, splits,
-                              G, n_pad, n, s1, b1, w2, b2, wc, bc, wm, bm, dest, debug_logits);
+                              G, n_pad, n, s1, b1, w2, b2, wc, bc, wm, bm, out_rows, debug_logits);
         if (n <= kSmallLaunch)
             return launch_pdl(head_rows_kernel<8>, dim3((n + 7) / 8), dim3(kThreadsRows), 0, s, partials, splits, G,
-                              n_pad, n, s1, b1, w2, b2, wc, bc, wm, bm, dest, debug_logits);
+                              n_pad, n, s1, b1, w2, b2, wc, bc, wm, bm, out_rows, debug_logits);
         return launch_pdl(head_rows_kernel<32>, dim3((n + 31) / 32), dim3(kThreadsRows), 0, s, partials, splits, G,
-                          n_pad, n, s1, b1, w2, b2, wc, bc, wm, bm, dest, debug_logits);
+                          n_pad, n, s1, b1, w2, b2, wc, bc, wm, bm, out_rows, debug_logits);
     }
     if (n > kSmallLaunch) {
         const long long tmo = (long long)timeout_ns;
         return launch_pdl(head_tile_kernel, dim3((n + kTileHits - 1) / kTileHits), dim3(kThreadsTile), kTileSmem, s,
-                          partials, splits, G, n_pad, n, s1, b1, w2, b2, wc, bc, wm, bm, dest, debug_logits,
+                          partials, splits, G, n_pad, n, s1, b1, w2, b2, wc, bc, wm, bm, out_rows, debug_logits,
                           head_counts_tiles(n, G) ? tile_done : nullptr, status, tmo);
     }
     return launch_pdl(head_kernel, dim3((n + kThreadsHead - 1) / kThreadsHead), dim3(kThreadsHead), 0, s, partials,
-                      splits, G, n_pad, n, s1, b1, w2, b2, wc, bc, wm, bm, dest, debug_logits);
+                      splits, G, n_pad, n, s1, b1, w2, b2, wc, bc, wm, bm, out_rows, debug_logits);
 }
 
 }  // namespace emtk
