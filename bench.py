@@ -37,8 +37,8 @@ METRIC = "hit patches/sec on 1 GB300 (extract+CNN); % bf16 tensor peak; gather H
 # precision, each from one ncu capture of this benchmark (profiles/launch_list_full_event_*.md),
 # with the kernel source it was taken on: reported as null once that source changes.
 TC_TRAFFIC = {
-    "bf16": (51_318_272 + 9_435_648, "cnn_tc.cu", "1c164a076dd4890c"),
-    "fp8": (38_921_216 + 3_531_520, "cnn_tc.cu", "1c164a076dd4890c"),
+    "bf16": (51_517_440 + 9_344_512, "cnn_tc.cu", "d9c50f1f72130cf7"),
+    "fp8": (38_985_728 + 3_194_880, "cnn_tc.cu", "d9c50f1f72130cf7"),
     "tf32": (979_775_744 + 435_545_600, "cnn_split.cu", "b3b11cc28934b03a"),
 }
 
