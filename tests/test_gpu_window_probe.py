@@ -29,7 +29,7 @@ pixels; the oracle's own fp64 network on the same weights must agree too
 (a check of the test's decoding).  Across the contexts every pixel of the
 window is probed, through taps that vary over all 25, for hits at every
 phase of the image row (e0 % 8), hits whose window reaches into the zero
-border, hits outside the plane, and, once, through pre-cut patches.
+border, hits outside the plane, and through pre-cut patches.
 
 Each probe runs twice: alone (a small launch, whose interval image is built
 from the whole plane) and batched with a 105.6 MB plane holding one hit (a
@@ -196,10 +196,9 @@ def test_window_read_bit_exact(emtk, big, prec):
             emtk.emtk_infer_batch(ctx, [(db, NT, db_hits, db_out), (big_adc, BIG_NT, big_hits, big_out)])
             tiled = torch.full((n, 8), float("nan"), dtype=torch.float32, device="cuda")
             emtk.emtk_infer_batch(ctx, [(adc, NT, hits, tiled), (big_adc, BIG_NT, big_hits, big_out)])
-            via_patches = None
-            if gi == 0:                    # the pre-cut patch path reads the same windows
-                via_patches = torch.full((n, 8), float("nan"), dtype=torch.float32, device="cuda")
-                emtk.emtk_infer_patches(ctx, patches, via_patches)
+            # the pre-cut patch path reads the same windows (from the fp32 patches themselves)
+            via_patches = torch.full((n, 8), float("nan"), dtype=torch.float32, device="cuda")
+            emtk.emtk_infer_patches(ctx, patches, via_patches)
             assert emtk.emtk_check(ctx) == emtk.EMTK_OK
         finally:
             emtk.emtk_destroy(ctx)
@@ -214,8 +213,56 @@ def test_window_read_bit_exact(emtk, big, prec):
         assert bad.size == 0, (f"{prec}, tiled cut, pixel group {gi}: {len(bad)} logits differ, first at hit "
                                f"{hits_np[bad[0][0]].tolist()} logit {bad[0][1]}: {got_t[tuple(bad[0])]} "
                                f"!= {want[tuple(bad[0])]}")
-        if via_patches is not None:
-            assert np.array_equal(via_patches[:, 4:].cpu().numpy().astype(np.float64), want)
+        assert np.array_equal(via_patches[:, 4:].cpu().numpy().astype(np.float64), want), \
+            f"{prec}, pre-cut patches, pixel group {gi}"
         if gi % 16 == 0:                   # the oracle's own network on these weights gives the same sums
             lo, _ = oracle.forward(want_p, w)
             assert np.array_equal(lo, want)
+
+
+def rounding_patches(n, fmt, seed):
+    """Positive fp32 patch values (the conv's ReLU keeps them) that need rounding
+    to 16 bit: random ones, and as many exact halfway cases of the format, with
+    the kept part's last bit even and odd."""
+    rng = np.random.default_rng(seed)
+    x = np.exp2(rng.uniform(-6.0, 10.0, (n, 48, 48))).astype(np.float32)
+    b = x.view(np.uint32)
+    tie = rng.random((n, 48, 48)) < 0.5
+    if fmt == "bf16":   # 16 dropped bits: halfway is 0x8000
+        b[tie] = (b[tie] & np.uint32(0xFFFF0000)) | np.uint32(0x8000)
+    else:               # fp16 keeps 10 of fp32's 23 mantissa bits here: halfway is 0x1000
+        b[tie] = (b[tie] & np.uint32(0xFFFFE000)) | np.uint32(0x1000)
+    return b.view(np.float32)
+
+
+@pytest.mark.parametrize("prec", ["bf16", "fp16"])
+def test_precut_patch_rounding_bit_exact(emtk, prec):
+    """The 16-bit network kernels round pre-cut fp32 patches as they load them:
+    to nearest, ties to even, as the oracle's rounding.  With one pixel per logit
+    (weights as in the window probe, the dense-1 weight 2^-8), each logit is
+    2^-8 times that pixel rounded, exactly."""
+    n = 300
+    x = rounding_patches(n, prec, seed=93 if prec == "bf16" else 94)
+    if prec == "bf16":
+        r = (oracle.round_bf16(x).astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    else:
+        r = oracle.round_fp16(x).astype(np.float64)
+    assert (r != x).mean() > 0.5      # most values are changed by the rounding
+    xd = torch.from_numpy(x).cuda()
+    groups = probe_pixels(1)[::48]     # 12 contexts of 4 pixels, spread over the window
+    for gi, pixels in enumerate(groups):
+        w, where = probe_weights(pixels, 1)
+        ctx = emtk.emtk_create(w, precision=prec, debug_logits=True, max_hits=512)
+        try:
+            out = torch.full((n, 8), float("nan"), dtype=torch.float32, device="cuda")
+            emtk.emtk_infer_patches(ctx, xd, out)
+            assert emtk.emtk_check(ctx) == emtk.EMTK_OK
+        finally:
+            emtk.emtk_destroy(ctx)
+        got = out[:, 4:].cpu().numpy().astype(np.float64)
+        want = np.zeros((n, 4))
+        for L, k, rr, cc in where:
+            want[:, L] += 2.0 ** (4 * k - 8) * r[:, rr, cc]
+        bad = np.argwhere(got != want)
+        assert bad.size == 0, (f"{prec}, group {gi}: {len(bad)} logits differ, first hit {bad[0][0]} logit "
+                               f"{bad[0][1]}: {got[tuple(bad[0])]} != {want[tuple(bad[0])]}")
