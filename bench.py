@@ -657,8 +657,8 @@ def run_sweep(args, rank, world, local_rank):
 HITFIND_THRESHOLD = 15.0  # 5 sigma of the synthetic planes' noise
 # DRAM bytes (read + write) of one hf_find_kernel launch on the full event, from one ncu
 # capture of this workload (profiles/hitfind_full_event.md); null once hitfind.cu changes.
-HF_TRAFFIC_BYTES = 369_249_280 + 4_627_200
-HF_TRAFFIC_SOURCE_SHA256 = "cd011a8a1983c3a1"
+HF_TRAFFIC_BYTES = 369_188_864 + 4_362_496
+HF_TRAFFIC_SOURCE_SHA256 = "2ba949573c38cacd"
 
 
 def hf_traffic():

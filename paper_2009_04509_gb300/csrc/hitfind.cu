@@ -44,7 +44,7 @@
 namespace emtk {
 namespace {
 
-constexpr int kHfWarps = 8;     // warps (units) per CTA of the find kernel
+constexpr int kHfWarps = 4;     // warps (units) per CTA of the find kernel
 constexpr int kHfSub = 4;       // 128-tick blocks loaded per step (4 loads in flight per lane)
 constexpr int kRunSlots = 128;  // runs per unit kept in scratch (more: the unit is scanned again)
 constexpr int kHfChunk = 128;   // units per chunk: threads per CTA of the place kernel
@@ -162,10 +162,15 @@ __device__ __forceinline__ int32_t scan_unit(const Unit &un, Src src, int nticks
         float4 v[kHfSub];
 #pragma unroll
         for (int k = 0; k < kHfSub; ++k) v[k] = src.group(base + 128 * k + 4 * lane);
-        float mx = -INFINITY;  // fmaxf skips NaN, which is never above
+        // fmaxf skips NaN, which is never above
+        bool hot[kHfSub];
+        bool any_hot = false;
 #pragma unroll
-        for (int k = 0; k < kHfSub; ++k) mx = fmaxf(mx, fmaxf(fmaxf(v[k].x, v[k].y), fmaxf(v[k].z, v[k].w)));
-        if (!__any_sync(kFull, mx > thr)) {
+        for (int k = 0; k < kHfSub; ++k) {
+            hot[k] = fmaxf(fmaxf(v[k].x, v[k].y), fmaxf(v[k].z, v[k].w)) > thr;
+            any_hot = any_hot || hot[k];
+        }
+        if (!__any_sync(kFull, any_hot)) {
             before = -INFINITY;  // the stretch's last tick is below
             continue;
         }
@@ -177,6 +182,10 @@ __device__ __forceinline__ int32_t scan_unit(const Unit &un, Src src, int nticks
         src.send = base + 128 * kHfSub < un.t1 ? base + 128 * kHfSub : un.t1;
 #pragma unroll
         for (int k = 0; k < kHfSub; ++k) {
+            if (!__any_sync(kFull, hot[k])) {  // no tick of the block is above: no start, no run end
+                before = -INFINITY;
+                continue;
+            }
             const float x[4] = {v[k].x, v[k].y, v[k].z, v[k].w};
             const bool a[4] = {x[0] > thr, x[1] > thr, x[2] > thr, x[3] > thr};
             const uint32_t b3 = __ballot_sync(kFull, a[3]);
