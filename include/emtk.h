@@ -155,10 +155,13 @@ typedef enum {
 } emtk_kernel;
 
 typedef struct {
+    /* launches: kernels of this library launched (a tiled patch cut and a
+     * hit-finding group are two each); chunks: network launches */
     uint64_t calls, hits, launches, chunks;
     uint64_t batch_hist[8];   /* hits per launch: <256, <1k, <2k, <4k, <8k, <16k, <64k, >=64k */
-    /* with options.profile: launches and summed device milliseconds per
-     * kernel class (emtk_get_stats waits for the recorded events) */
+    /* kernels launched per kernel class and, with options.profile, summed
+     * device milliseconds per class (emtk_get_stats waits for the recorded
+     * events; a class's time spans all its kernels of one call) */
     uint64_t kernel_launches[EMTK_NUM_KERNELS];
     double kernel_ms[EMTK_NUM_KERNELS];
 } emtk_stats;

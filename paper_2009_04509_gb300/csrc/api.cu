@@ -121,18 +121,18 @@ const char *const kNvtxNames[EMTK_NUM_KERNELS] = {"emtk interval images (patch c
                                                   "emtk network (conv + dense-1)", "emtk head (dense-2 + heads)",
                                                   "emtk convert patches", "emtk hit finding"};
 
-// Around one launch: an NVTX range on the host thread (always; free unless a
-// profiler is attached) and, in profile mode, CUDA events on the caller's
-// stream.
+// Around the launch of `kernels` kernels of one class: an NVTX range on the
+// host thread (always; free unless a profiler is attached), the launch counts
+// and, in profile mode, CUDA events on the caller's stream.
 struct Prof {
     emtk_ctx *c;
     int kind;
     cudaStream_t s;
     cudaEvent_t a = nullptr, b = nullptr;
-    Prof(emtk_ctx *c_, int kind_, cudaStream_t s_) : c(c_), kind(kind_), s(s_) {
+    Prof(emtk_ctx *c_, int kind_, cudaStream_t s_, int kernels = 1) : c(c_), kind(kind_), s(s_) {
         nvtxRangePushA(kNvtxNames[kind]);
-        c->stats.launches++;
-        c->stats.kernel_launches[kind]++;
+        c->stats.launches += (uint64_t)kernels;
+        c->stats.kernel_launches[kind] += (uint64_t)kernels;
         if (!c->opt.profile) return;
         if (cudaEventCreate(&a) != cudaSuccess || cudaEventCreate(&b) != cudaSuccess) {
             if (a) cudaEventDestroy(a);
@@ -323,7 +323,7 @@ emtk_status run_requests(emtk_ctx *c, const emtk_request *reqs, int32_t nreq, cu
             // first chunk's window descriptors are built in the same launch
             const DescJob job{0, (int32_t)std::min<int64_t>(c->max_hits, hits), c->ws.hdesc, c->ws.dest,
                               out_stride(c)};
-            Prof prof(c, EMTK_KERNEL_INTERVALS, s);
+            Prof prof(c, EMTK_KERNEL_INTERVALS, s, tiles ? 2 : 1);  // the tiled cut: marks, then tiles
             if (tiles) {
                 uint32_t *cur = c->tile_mask + (int64_t)c->tile_mask_parity * c->tile_mask_cap;
                 uint32_t *next = c->tile_mask + (int64_t)(1 - c->tile_mask_parity) * c->tile_mask_cap;
@@ -840,7 +840,7 @@ emtk_status emtk_find_hits(emtk_ctx *c, emtk_hitfind_request *reqs, int32_t nreq
         int32_t *cur = c->hf_sums + (int64_t)c->hf_parity * c->hf_sums_cap;
         int32_t *next = c->hf_sums + (int64_t)(1 - c->hf_parity) * c->hf_sums_cap;
         {
-            Prof prof(c, EMTK_KERNEL_HITFIND, s);
+            Prof prof(c, EMTK_KERNEL_HITFIND, s, U > 0 ? 2 : 0);  // find, then place
             e = launch_find_hits(t, U, scratch, cur, next, c->hf_sums_cap, totals, s);
         }
         if (e == cudaSuccess && U > 0) c->hf_parity ^= 1;

@@ -176,3 +176,33 @@ def test_full_event_patch_cut_bit_exact(emtk, event):
             assert np.array_equal(b16.cpu().numpy().view(np.uint16), oracle.round_bf16(want))
     finally:
         emtk.emtk_destroy(ctx)
+
+
+def test_launch_counts(emtk, event):
+    """The library's launch count is the number of its kernels launched: a
+    full-event call is four (tile marks, the touched image tiles with the window
+    descriptors, the network, the head), a small single-plane call three (the
+    whole-plane images with the descriptors, the network, the head), and a
+    hit-finding call two (find, place)."""
+    planes = event["planes"]
+    ctx = emtk.emtk_create(event["weights"], precision="bf16")
+    try:
+        items = [(torch.from_numpy(p.adc).cuda(), p.nticks, torch.from_numpy(p.hits).cuda(),
+                  torch.empty((p.nhits, 4), device="cuda")) for p in planes]
+        base = emtk.emtk_get_stats(ctx)["launches"]
+        emtk.emtk_infer_batch(ctx, items)
+        assert emtk.emtk_check(ctx) == emtk.EMTK_OK
+        assert emtk.emtk_get_stats(ctx)["launches"] - base == 4
+        adc, nticks, hits, _ = items[2]
+        small = torch.empty((256, 4), device="cuda")
+        base = emtk.emtk_get_stats(ctx)["launches"]
+        emtk.emtk_infer(ctx, adc, nticks, hits[:256], small)
+        assert emtk.emtk_check(ctx) == emtk.EMTK_OK
+        assert emtk.emtk_get_stats(ctx)["launches"] - base == 3
+        cap = 65536
+        req = [(adc, nticks, 15.0, torch.empty((cap, 2), dtype=torch.int32, device="cuda"), None)]
+        base = emtk.emtk_get_stats(ctx)["launches"]
+        emtk.emtk_find_hits(ctx, req)
+        assert emtk.emtk_get_stats(ctx)["launches"] - base == 2
+    finally:
+        emtk.emtk_destroy(ctx)
