@@ -597,26 +597,21 @@ emtk_status emtk_infer_patches(emtk_ctx *c, const float *d_patches, int32_t n, f
     for (int64_t h0 = 0; h0 < n && st == EMTK_OK; h0 += c->max_hits) {
         const int32_t cnt = (int32_t)std::min<int64_t>(c->max_hits, n - h0);
         const float *src = d_patches + h0 * kPatchElems;
-        const void *net_in = src;
-        float *rows = d_scores + h0 * out_stride(c);
+        // the head writes hit h's scores to rows + h * stride (no pointer table)
+        const OutRows out{nullptr, d_scores + h0 * out_stride(c), out_stride(c)};
         if (fmt == EMTK_PATCH_BF16 || fmt == EMTK_PATCH_F16) {
-            // the tensor-core kernel reads the fp32 patches itself (no conversion launch), and
-            // the head writes each hit's scores to rows + h * stride
-            st = run_network(c, nullptr, nullptr, cnt, OutRows{nullptr, rows, out_stride(c)}, src, s);
-            continue;
-        }
-        {
-            // the patches in the network's format and each hit's output row, in one launch
-            Prof prof(c, EMTK_KERNEL_CONVERT, s);
-            if (fmt != EMTK_PATCH_F32) {
-                st = cuda_status(launch_convert_patches(src, c->ws.patches, fmt, (int64_t)cnt * kPatchElems, rows,
-                                                        out_stride(c), c->ws.dest, cnt, c->sm_count, s));
-                net_in = c->ws.patches;
-            } else {
-                st = cuda_status(launch_fill_dest(rows, out_stride(c), c->ws.dest, cnt, s));
+            // the tensor-core kernel reads the fp32 patches itself: no conversion launch
+            st = run_network(c, nullptr, nullptr, cnt, out, src, s);
+        } else if (fmt == kPatchSplit16) {
+            {
+                // the split-fp16 network reads head / tail words: one conversion launch first
+                Prof prof(c, EMTK_KERNEL_CONVERT, s);
+                st = cuda_status(launch_convert_split(src, c->ws.patches, (int64_t)cnt * kPatchElems, c->sm_count, s));
             }
+            if (st == EMTK_OK) st = run_network(c, c->ws.patches, nullptr, cnt, out, nullptr, s);
+        } else {
+            st = run_network(c, src, nullptr, cnt, out, nullptr, s);  // the fp32 kernel reads the patches
         }
-        if (st == EMTK_OK) st = run_network(c, net_in, nullptr, cnt, OutRows{c->ws.dest, nullptr, 0}, nullptr, s);
     }
     c->stats.calls++;
     c->stats.hits += (uint64_t)n;

@@ -278,15 +278,13 @@ cudaError_t launch_cut_tiles(const ReqTable &t, int64_t total_hits, void *dimg, 
 cudaError_t launch_gather(const ReqTable &t, const void *dimg, emtk_patch_format fmt, int64_t g0,
                           int32_t count, void *patches, float **dest, int out_stride, cudaStream_t s);
 // Pre-cut fp32 patches (n values, a multiple of 8, 16-byte aligned) into the
-// network's patch format at dst, and dest[i] = scores + i * out_stride for
-// the nhits hits, in one launch of at most 8 CTAs per SM.
-cudaError_t launch_convert_patches(const float *src, void *dst, emtk_patch_format fmt, int64_t n, float *scores,
-                                   int out_stride, float **dest, int32_t nhits, int sms, cudaStream_t s);
+// split-fp16 head / tail words of the EMTK_TF32 network at dst (n words), in
+// one launch of at most 8 CTAs per SM.
+cudaError_t launch_convert_split(const float *src, void *dst, int64_t n, int sms, cudaStream_t s);
 // Window descriptors of hits [g0, g0+count) (images with halo kHalo), and
 // the output row of each hit in dest.
 cudaError_t launch_hit_desc(const ReqTable &t, int64_t g0, int32_t count, HitDesc *desc, float **dest,
                             int out_stride, cudaStream_t s);
-cudaError_t launch_fill_dest(float *scores, int out_stride, float **dest, int32_t n, cudaStream_t s);
 // Hit finding of the group's planes (hitfind.cu): scratch (256-byte aligned)
 // holds per-unit run counts and run slots; find_hits_unit_cap gives the most
 // units that scratch_bytes holds.  The chunk sums live in sums_cur (zero on

@@ -185,19 +185,16 @@ __global__ void __launch_bounds__(288) gather_kernel(const __grid_constant__ Req
     }
 }
 
-// Pre-cut fp32 patches -> the network's patch format (emtk_infer_patches):
-// eight values per thread and step (two 16-byte streaming loads, so the
-// dense-1 weights keep their place in L2), four steps in flight; the same
-// rounding per value as the interval images (RNE to 16 bit, or the split
-// head / tail word).  The first threads also write each hit's output row.
-// n8 = values / 8 (a patch is 2,304 values).
-template <int FMT>
-__global__ void convert_kernel(const float *__restrict__ src, void *__restrict__ dst, int64_t n8,
-                               float *scores, int stride, float **dest, int32_t nhits) {
+// Pre-cut fp32 patches -> the split-fp16 head / tail words of the EMTK_TF32
+// network (emtk_infer_patches; the 16-bit kernels read fp32 patches
+// themselves): eight values per thread and step (two 16-byte streaming loads,
+// so the dense-1 weights keep their place in L2), four steps in flight; the
+// same word per value as the interval images.  n8 = values / 8 (a patch is
+// 2,304 values).
+__global__ void convert_split_kernel(const float *__restrict__ src, uint4 *__restrict__ dst, int64_t n8) {
     pdl_trigger();  // the network kernel may set up while this one runs; it waits for it
     const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const int64_t nthreads = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t i = tid; i < nhits; i += nthreads) dest[i] = scores + i * stride;
     const float4 *s4 = reinterpret_cast<const float4 *>(src);
     constexpr int kU = 4;
     for (int64_t base = tid; base < n8; base += nthreads * kU) {
@@ -214,25 +211,9 @@ __global__ void convert_kernel(const float *__restrict__ src, void *__restrict__
         for (int u = 0; u < kU; ++u) {
             const int64_t i = base + u * nthreads;
             if (i >= n8) continue;
-            const float v[8] = {a[u].x, a[u].y, a[u].z, a[u].w, b[u].x, b[u].y, b[u].z, b[u].w};
-            if (FMT == kPatchSplit16) {
-                uint4 *d = static_cast<uint4 *>(dst) + 2 * i;
-                d[0] = make_uint4(split_word(v[0]), split_word(v[1]), split_word(v[2]), split_word(v[3]));
-                d[1] = make_uint4(split_word(v[4]), split_word(v[5]), split_word(v[6]), split_word(v[7]));
-            } else {
-                uint32_t w[4];
-#pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    if (FMT == EMTK_PATCH_BF16) {
-                        const __nv_bfloat162 h = __floats2bfloat162_rn(v[2 * k], v[2 * k + 1]);
-                        w[k] = *reinterpret_cast<const uint32_t *>(&h);
-                    } else {
-                        const __half2 h = __floats2half2_rn(v[2 * k], v[2 * k + 1]);
-                        w[k] = *reinterpret_cast<const uint32_t *>(&h);
-                    }
-                }
-                static_cast<uint4 *>(dst)[i] = make_uint4(w[0], w[1], w[2], w[3]);
-            }
+            dst[2 * i] = make_uint4(split_word(a[u].x), split_word(a[u].y), split_word(a[u].z), split_word(a[u].w));
+            dst[2 * i + 1] =
+                make_uint4(split_word(b[u].x), split_word(b[u].y), split_word(b[u].z), split_word(b[u].w));
         }
     }
 }
@@ -425,12 +406,6 @@ __global__ void __launch_bounds__(kTileWarps * 32) interval_tiles_kernel(const _
     }
 }
 
-__global__ void fill_dest_kernel(float *scores, int stride, float **dest, int32_t n) {
-    pdl_trigger();
-    const int i = blockIdx.x * blockDim.x + threadIdx.x;
-    if (i < n) dest[i] = scores + (int64_t)i * stride;
-}
-
 }  // namespace
 
 cudaError_t launch_interval_images(const ReqTable &t, void *dimg, emtk_patch_format fmt, cudaStream_t s,
@@ -531,19 +506,13 @@ cudaError_t launch_gather(const ReqTable &t, const void *dimg, emtk_patch_format
     return cudaGetLastError();
 }
 
-cudaError_t launch_convert_patches(const float *src, void *dst, emtk_patch_format fmt, int64_t n, float *scores,
-                                   int out_stride, float **dest, int32_t nhits, int sms, cudaStream_t s) {
+cudaError_t launch_convert_split(const float *src, void *dst, int64_t n, int sms, cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
     const int64_t n8 = n / 8;
     int64_t blocks = (n8 + 256 * 4 - 1) / (256 * 4);
     if (blocks > (int64_t)sms * 8) blocks = (int64_t)sms * 8;
     if (blocks < 1) blocks = 1;
-    if (fmt == kPatchSplit16)
-        convert_kernel<kPatchSplit16><<<(unsigned)blocks, 256, 0, s>>>(src, dst, n8, scores, out_stride, dest, nhits);
-    else if (fmt == EMTK_PATCH_BF16)
-        convert_kernel<EMTK_PATCH_BF16><<<(unsigned)blocks, 256, 0, s>>>(src, dst, n8, scores, out_stride, dest, nhits);
-    else
-        convert_kernel<EMTK_PATCH_F16><<<(unsigned)blocks, 256, 0, s>>>(src, dst, n8, scores, out_stride, dest, nhits);
+    convert_split_kernel<<<(unsigned)blocks, 256, 0, s>>>(src, static_cast<uint4 *>(dst), n8);
     return cudaGetLastError();
 }
 
@@ -551,12 +520,6 @@ cudaError_t launch_hit_desc(const ReqTable &t, int64_t g0, int32_t count, HitDes
                             int out_stride, cudaStream_t s) {
     if (count <= 0) return cudaSuccess;
     hit_desc_kernel<<<(count + 255) / 256, 256, 0, s>>>(t, g0, count, desc, dest, out_stride);
-    return cudaGetLastError();
-}
-
-cudaError_t launch_fill_dest(float *scores, int out_stride, float **dest, int32_t n, cudaStream_t s) {
-    if (n <= 0) return cudaSuccess;
-    fill_dest_kernel<<<(n + 255) / 256, 256, 0, s>>>(scores, out_stride, dest, n);
     return cudaGetLastError();
 }
 
