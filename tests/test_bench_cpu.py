@@ -66,3 +66,29 @@ def test_network_peaks():
     assert abs(bench.network_peak("tf32", peaks)[0] - 1900.0 / 3.0) < 1e-9
     p32, src = bench.network_peak("fp32", peaks)
     assert abs(p32 - 152 * 128 * 2 * 2.07e9 / 1e12) < 1e-9 and "derived" in src
+
+
+def test_tiled_cut_label_follows_the_library_threshold():
+    """The benchmark names the patch-cut kernels from the planes' size with the
+    library's rule: the tiled cut from 96 MiB of planes with hits.  The
+    threshold is read from the library source so that the two cannot drift."""
+    import os
+    import re
+    src = open(os.path.join(os.path.dirname(bench.__file__), "paper_2009_04509_gb300", "csrc", "api.cu")).read()
+    m = re.search(r"constexpr int64_t kTiledCutMinBytes = \(int64_t\)(\d+) << (\d+);", src)
+    assert m, "the threshold's definition moved"
+    limit = int(m.group(1)) << int(m.group(2))
+    words = limit // 4
+
+    class P:  # a plane of `nwires` x 6000 fp32 ticks with or without hits
+        def __init__(self, nwires, nhits):
+            self.nwires, self.nticks, self.nhits = nwires, 6000, nhits
+
+    at = -(-words // 6000)   # wires that just reach the threshold
+    assert bench.tiled_cut([P(at, 1)])
+    assert not bench.tiled_cut([P(at - 1, 1)])
+    assert not bench.tiled_cut([P(at, 0)])                  # planes without hits do not count
+    assert bench.tiled_cut([P(at // 2, 3), P(at - at // 2, 5)])
+    full = synth.full_event(seed=0)
+    assert bench.tiled_cut(full)                              # 368.6 MB: the tiled cut
+    assert not bench.tiled_cut([synth.single_plane(seed=0)])  # 11.5 MB: whole planes
